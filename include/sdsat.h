@@ -1,0 +1,257 @@
+/*
+ * libsdsat -- the SDSAT block decode step on one GB300 (sm_103a).
+ *
+ * SDSAT ("Speculative Decoding with Semantic Adaptive Tokens", arXiv
+ * 2403.18647) decodes with an unmodified Llama-architecture model in loops of
+ * "two-step-draft-then-verify" (Sec. 2.1):
+ *
+ *   draft step 1 (Eq. 1)  block [last token, a_1 .. a_k]  -> y_{n+1} and k drafts
+ *   draft step 2 (Eq. 2)  block [y_{n+1}, d_1 .. d_k]     -> targets t_0 .. t_k
+ *   verification (Eq. 3)  accept t_0 .. t_m, m = leading matches d_i == t_{i-1}
+ *
+ * Each step is one pass of q = k + 1 positions through every layer
+ * (sdsat_block_forward), then target selection, verification and KV commit
+ * (sdsat_accept_greedy / sdsat_accept_nucleus).  The loop emits 2 + m tokens
+ * for two passes (Sec. 2.1.1).
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ *  - Pointers named *_dev are CUDA device pointers owned by the caller; they
+ *    must stay valid until the work queued on the context stream has run.
+ *  - All compute calls are asynchronous on the context stream
+ *    (sdsat_set_stream); only sdsat_create, sdsat_kv_create, sdsat_*_destroy
+ *    and sdsat_get_error synchronise.  No compute call allocates memory, so
+ *    compute calls may be captured into a CUDA graph.
+ *  - Argument errors are detected on the host and returned synchronously
+ *    (nothing is queued).  Errors only the device can see (a NaN logit, a
+ *    row past the KV capacity, a timed-out wait) set bits in a device flag
+ *    word read by sdsat_get_error.
+ *  - Weights are bf16, row-major [out_features, in_features] (the layout of
+ *    nn.Linear.weight), 16-byte aligned, in_features a multiple of 8.
+ *  - Activations and logits are fp32; token ids int32.
+ */
+#ifndef SDSAT_H
+#define SDSAT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SDSAT_API __attribute__((visibility("default")))
+#else
+#define SDSAT_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SDSAT_OK = 0,
+  SDSAT_EINVAL = 1,        /* bad argument: null/misaligned pointer, size out of range */
+  SDSAT_ENOMEM = 2,        /* device allocation failed (create calls only) */
+  SDSAT_ECAPACITY = 3,     /* batch, q, position or KV capacity limit exceeded */
+  SDSAT_ECUDA = 4,         /* a CUDA runtime or driver call failed */
+  SDSAT_EDEVICE = 5,       /* device-detected error bits were set (sdsat_get_error) */
+  SDSAT_EUNSUPPORTED = 6   /* a configuration this build does not implement */
+} sdsat_status;
+
+/* device error bits reported by sdsat_get_error */
+#define SDSAT_DEV_NAN_LOGITS 0x1u  /* NaN logit seen; it counted as -inf */
+#define SDSAT_DEV_TIMEOUT 0x2u     /* a bounded in-kernel wait expired; results invalid */
+#define SDSAT_DEV_CAPACITY 0x4u    /* a block row fell past the KV capacity; not written */
+#define SDSAT_DEV_TOKEN 0x8u       /* a token id outside [0, vocab); id 0 used instead */
+#define SDSAT_DEV_POSITION 0x10u   /* a RoPE position outside [0, max_position); clamped */
+
+#define SDSAT_MAX_Q 16           /* block rows per sequence (k <= 15 adaptive tokens) */
+#define SDSAT_MAX_ROWS 64        /* batch * q rows per block forward */
+#define SDSAT_MAX_ADAPTIVE 16
+
+typedef struct sdsat_ctx sdsat_ctx;
+typedef struct sdsat_kv sdsat_kv;
+
+/* Model and decoding configuration (Llama architecture; Sec. 3 uses CodeLlama). */
+typedef struct {
+  int32_t n_layers;
+  int32_t d_model;
+  int32_t n_heads;
+  int32_t n_kv_heads;      /* must equal n_heads in this build (no grouped-query attention) */
+  int32_t head_dim;        /* 64 or 128 */
+  int32_t ffn_dim;         /* SwiGLU hidden size */
+  int32_t vocab;           /* including the semantic adaptive tokens (Sec. 3.2: ordinary ids) */
+  float rms_eps;
+  float rope_theta;        /* RoPE base; rotate-half pairing (i, i + head_dim/2) */
+  int32_t max_position;    /* RoPE table length: every position must be < max_position */
+  int32_t n_adaptive;      /* 1: adaptive_ids[0] repeated k times (recommended, App. B);
+                              >1: k distinct ids a_1..a_k (SDSAT-D, App. B) */
+  int32_t adaptive_ids[SDSAT_MAX_ADAPTIVE];
+} sdsat_config;
+
+/* Per-layer weights (device pointers, borrowed: the caller keeps them alive). */
+typedef struct {
+  const void* attn_norm;   /* bf16 [d] */
+  const void* wq;          /* bf16 [H*hd, d] */
+  const void* wk;          /* bf16 [H*hd, d] */
+  const void* wv;          /* bf16 [H*hd, d] */
+  const void* wo;          /* bf16 [d, H*hd] */
+  const void* ffn_norm;    /* bf16 [d] */
+  const void* w_gate;      /* bf16 [F, d] */
+  const void* w_up;        /* bf16 [F, d] */
+  const void* w_down;      /* bf16 [d, F] */
+} sdsat_layer_weights;
+
+typedef struct {
+  const void* embed;                    /* bf16 [V, d] */
+  const void* final_norm;               /* bf16 [d] */
+  const void* lm_head;                  /* bf16 [V, d] (untied) */
+  const sdsat_layer_weights* layers;    /* host array of n_layers entries (copied) */
+} sdsat_weights;
+
+/* ---- lifetime ----------------------------------------------------------------- */
+
+/* Validate `cfg`, record the weight pointers, build the TMA descriptors and the
+ * RoPE table, allocate the library-owned workspaces.  `stream` is a cudaStream_t
+ * (NULL = legacy default stream).  Synchronous.  Errors: EINVAL (bad config or
+ * pointer), EUNSUPPORTED (head_dim, GQA), ENOMEM, ECUDA. */
+SDSAT_API sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void* stream,
+                          sdsat_ctx** out);
+SDSAT_API void sdsat_destroy(sdsat_ctx* ctx);
+
+/* Stream for all later compute calls on ctx (a cudaStream_t). */
+SDSAT_API sdsat_status sdsat_set_stream(sdsat_ctx* ctx, void* stream);
+
+/* Library-owned KV cache for `batch` sequences of up to `max_len` slots:
+ * K and V bf16 [n_layers][batch][n_heads][max_len][head_dim], and the committed
+ * length len[batch] (int32, device, starts at 0).  Synchronous.
+ * Errors: EINVAL, ENOMEM. */
+SDSAT_API sdsat_status sdsat_kv_create(sdsat_ctx* ctx, int batch, int max_len, sdsat_kv** out);
+SDSAT_API void sdsat_kv_destroy(sdsat_kv* kv);
+
+/* Device addresses and geometry of a KV cache (for tests and benches that fill
+ * or inspect it).  Any output pointer may be NULL. */
+SDSAT_API sdsat_status sdsat_kv_info(const sdsat_kv* kv, void** k_dev, void** v_dev, int32_t** len_dev,
+                           int* batch, int* max_len);
+
+/* Copy n rows into / out of the cache of one (layer, sequence), all heads:
+ * src / dst are bf16 [n_heads][n][head_dim] device buffers; rows land at slots
+ * slot0 .. slot0+n-1.  Asynchronous on the context stream.  Used to load a
+ * snapshot (or synthetic contents) and to inspect what a block forward wrote.
+ * Errors: EINVAL (null pointer, layer/seq/slot range). */
+SDSAT_API sdsat_status sdsat_kv_write(sdsat_ctx* ctx, sdsat_kv* kv, int layer, int seq, int slot0, int n,
+                                      const void* k_src_dev, const void* v_src_dev);
+SDSAT_API sdsat_status sdsat_kv_read(sdsat_ctx* ctx, const sdsat_kv* kv, int layer, int seq, int slot0, int n,
+                                     void* k_dst_dev, void* v_dst_dev);
+
+/* ---- the block decode step ------------------------------------------------------- */
+
+/* One pass of q new positions for sequences 0 .. b-1 through every layer
+ * (Eq. 1 and Eq. 2 evaluate P_theta at all q positions of a block at once).
+ *
+ * tokens_dev     int32 [b*q], row j of sequence s at s*q + j.
+ * positions_dev  int32 [b*q] RoPE positions, or NULL for len[s] + j.
+ * logits_dev     fp32 [b*q][vocab], written.
+ * Block rows are written to KV slots len[s] .. len[s]+q-1 (len is NOT advanced;
+ * see the accept calls and sdsat_kv_commit).  Row j attends to slots [0, len[s])
+ * and to block rows 0..j.
+ * Errors: EINVAL (null pointer, b < 1, b > kv batch, q < 1, q > SDSAT_MAX_Q,
+ * b*q > SDSAT_MAX_ROWS); device bit CAPACITY if len[s] + q > max_len. */
+SDSAT_API sdsat_status sdsat_block_forward(sdsat_ctx* ctx, sdsat_kv* kv, const int32_t* tokens_dev,
+                                 const int32_t* positions_dev, int b, int q, float* logits_dev);
+
+/* Greedy target selection, Eq. 3 verification and KV commit (Sec. 2.1.1).
+ *
+ * logits_dev        fp32 [b*q][vocab] from sdsat_block_forward.
+ * drafts_dev        int32 [b*q]: the block's input tokens; entry s*q + i (1 <= i < q)
+ *                   is draft d_i.  Entry s*q is not read.
+ * n_verify          number of drafts to verify (0 <= n_verify < q).  0 is draft
+ *                   step 1: only t_0 is emitted and rows 1..q-1 return the drafts.
+ * out_tokens_dev    int32 [b*q]: t_j = argmax of row j (lowest id on ties; NaN
+ *                   counts as -inf and sets device bit NAN_LOGITS), for every j.
+ * accepted_len_dev  int32 [b]: 1 + m, the number of emitted tokens t_0 .. t_m,
+ *                   m = max{i <= n_verify : d_i' == t_{i'-1} for all i' <= i}.
+ * commit            non-zero: len[s] += 1 + m on the device (rejected rows and
+ *                   the adaptive positions are rolled back by not committing them).
+ * Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_accept_greedy(sdsat_ctx* ctx, sdsat_kv* kv, const float* logits_dev,
+                                 const int32_t* drafts_dev, int b, int q, int n_verify,
+                                 int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit);
+
+/* Nucleus (top-p) variant (Sec. 2.1.2, chain form: the accepted branch is the
+ * longest verified prefix).  Each row's target is a sample defined exactly so
+ * that any two implementations agree bit for bit:
+ *   s_i = (l_i - max l) / temperature (fp32), w_i = exp(s_i) (fp32, Cody-Waite
+ *   reduction + degree-7 polynomial, every step one rounded operation),
+ *   W_i = floor(w_i * 2^40) (uint64);  candidates = the top_k heaviest by
+ *   (W desc, id asc) (top_k = 0: all);  kept = the shortest prefix of the
+ *   candidates in that order with C * 2^24 >= round(top_p * 2^24) * S;
+ *   r = Philox4x32-10(key = rng_seed, counter = (position of the produced
+ *   token, s, 0, 0)), 64-bit from its first two words;  tau = (r * S_kept) >> 64;
+ *   the sample is the first kept id, ascending, whose inclusive cumulative
+ *   weight exceeds tau.
+ * The produced token of row j has position len[s] + j + 1.  temperature <= 0
+ * selects greedy (Fig. 1: greedy is the special case).  Requires vocab <= 32768.
+ * Other arguments as sdsat_accept_greedy.  Errors: EINVAL, EUNSUPPORTED. */
+SDSAT_API sdsat_status sdsat_accept_nucleus(sdsat_ctx* ctx, sdsat_kv* kv, const float* logits_dev,
+                                  const int32_t* drafts_dev, int b, int q, int n_verify,
+                                  float top_p, float temperature, uint64_t rng_seed, int top_k,
+                                  int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit);
+
+/* Explicit commit / rollback: len[s] = new_len_dev[s] for s < b (device values,
+ * 0 <= new_len <= max_len; out-of-range values are clamped and set CAPACITY).
+ * Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_kv_commit(sdsat_ctx* ctx, sdsat_kv* kv, const int32_t* new_len_dev, int b);
+
+/* Copy the committed lengths len[0 .. b-1] into lens_dev (int32 [b], device),
+ * asynchronously.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_kv_lengths(sdsat_ctx* ctx, const sdsat_kv* kv, int32_t* lens_dev, int b);
+
+/* Build the next block input on the device (the block inputs of Eq. 1 and Eq. 2),
+ * so that a whole loop runs without the host:
+ *   mode 1 (draft step 1): row 0 = prev_out[s*q + prev_acc[s] - 1] (the newest
+ *     emitted token), rows 1..q-1 = the adaptive ids a_1 .. a_{q-1};
+ *   mode 2 (draft step 2): row 0 = prev_out[s*q] (y_{n+1}), rows 1..q-1 = the drafts:
+ *     prev_out[s*q + j] (the drafts draft step 1 produced), or, when
+ *     draft_table_dev is given, draft_table_dev[s*table_stride + len[s] + j]
+ *     (a per-position draft source, e.g. a test stub).
+ * prev_out_dev / prev_acc_dev are the out_tokens / accepted_len of the previous
+ * accept call; tokens_out_dev int32 [b*q] is written.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_build_block(sdsat_ctx* ctx, sdsat_kv* kv, int mode, const int32_t* prev_out_dev,
+                               const int32_t* prev_acc_dev, const int32_t* draft_table_dev,
+                               int table_stride, int b, int q, int32_t* tokens_out_dev);
+
+/* Run n prompt tokens of sequence `seq` through the model in blocks of up to
+ * SDSAT_MAX_Q rows and commit them (len[seq] += n).  No logits are produced.
+ * Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_prefill(sdsat_ctx* ctx, sdsat_kv* kv, int seq, const int32_t* tokens_dev, int n);
+
+/* Synchronise the context stream, return the accumulated device error bits in
+ * *flags (SDSAT_DEV_*) and clear them.  Returns EDEVICE if any bit was set,
+ * ECUDA if the stream reported a CUDA error. */
+SDSAT_API sdsat_status sdsat_get_error(sdsat_ctx* ctx, uint32_t* flags);
+
+SDSAT_API const char* sdsat_status_string(sdsat_status s);
+
+/* ---- single kernels (unit parity tests and kernel sweeps) ------------------------- */
+
+/* y[m][n] = sum_k x[m][k] * W[n][k] for m < M, n < N: the weight-streaming skinny
+ * GEMM behind every projection of the block forward.  x fp32 [M][K] (row stride
+ * K), W bf16 [N][K], y fp32 [M][N].  M <= SDSAT_MAX_ROWS.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_op_gemm(sdsat_ctx* ctx, const float* x_dev, int M, int K, const void* w_dev, int N,
+                           float* y_dev);
+
+/* Block-causal attention of q query rows per sequence against a bf16 cache:
+ * out[s*q+j][h*hd+d] = sum_t softmax_t(q_j . k_t / sqrt(hd)) v_t[d] over slots
+ * t < len[s] + j + 1.  q_dev fp32 [b*q][H*hd]; k_dev, v_dev bf16
+ * [b][H][cap][hd]; len_dev int32 [b] (device); out_dev fp32 [b*q][H*hd].
+ * hd must be 64 or 128.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, const void* k_dev, const void* v_dev,
+                                const int32_t* len_dev, int b, int q, int H, int hd, int cap,
+                                float* out_dev);
+
+/* out[i] = the nucleus sampler's exp (see sdsat_accept_nucleus) of in[i] <= 0. */
+SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* out_dev, int n);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SDSAT_H */

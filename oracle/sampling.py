@@ -13,8 +13,12 @@ a CPU and a GPU reach the same token from the same logits bit for bit:
   1. s_i = (l_i - max_j l_j) / T           one fp32 IEEE division
   2. w_i = exp_sd(s_i)                      fp32, every step a single
                                             correctly rounded operation
-  3. W_i = floor(w_i * 2^40)                exact uint64 weights; the
-                                            argmax has W = 2^40
+  3. W_i = floor(w_i * 2^24)                exact integer weights; the
+                                            argmax has W = 2^24.  A token
+                                            whose weight is below 2^-24 of
+                                            the top one gets W = 0: it is
+                                            below the resolution of an fp32
+                                            normaliser that already holds 1
   4. candidates: all ids, or the top_k largest by (W desc, id asc)
   5. kept set: the shortest prefix of the candidates in (W desc, id asc)
      order whose cumulative weight C satisfies C * 2^24 >= P * S, where
@@ -47,7 +51,7 @@ LN2_LO = f32(0.6931471805599453 - 0.693145751953125)
 EXP_COEF = [f32(1.0 / 5040.0), f32(1.0 / 720.0), f32(1.0 / 120.0), f32(1.0 / 24.0),
             f32(1.0 / 6.0), f32(0.5), f32(1.0), f32(1.0)]   # 1/7! ... 1/0!
 EXP_MIN = f32(-87.0)
-W_SHIFT = 40
+W_SHIFT = 24
 P_SHIFT = 24
 
 M32 = 0xFFFFFFFF
@@ -151,7 +155,7 @@ def nucleus_sample(logits: np.ndarray, temperature: float, top_p: float, seed: i
         C += int(W[i])
         if C > tau:
             return int(i), nan
-    return int(kept[-1]), nan                             # unreachable: C ends at S_kept > tau
+    return int(kept[-1]), nan       # only when S_kept == 0 (an all-NaN row): its single kept id
 
 
 def select(logits: np.ndarray, temperature: float = 0.0, top_p: float = 1.0, seed: int = 0,

@@ -1,0 +1,492 @@
+// Target selection, verification and KV commit, plus the small kernels of the
+// step (embedding gather, block-input building, explicit commit).
+//
+// Verification (Sec. 2.1.1, Eq. 3): with targets t_j (argmax or nucleus sample
+// of block row j) and drafts d_i (the block's input token of row i), draft i is
+// accepted while d_i == t_{i-1} for all i' <= i; the first mismatch stops the
+// loop.  The emitted tokens are t_0 .. t_m and the committed KV length grows by
+// 1 + m (the rejected rows, and in draft step 1 the adaptive-token rows, are
+// rolled back by not being committed).
+//
+// One CTA per block row selects that row's target; the last CTA of a sequence
+// (per-sequence counter, no waiting) runs the prefix scan and the commit.
+#include "common.cuh"
+#include "internal.h"
+
+namespace sdsat {
+
+// ---- the nucleus sampler's arithmetic -------------------------------------------
+// exp(s) for s <= 0: Cody-Waite reduction with a two-part ln 2, degree-7 Taylor
+// polynomial on |r| <= ln2/2 by Horner's rule, exact scaling by 2^n; every step
+// is one correctly rounded fp32 operation (no contraction), so any IEEE
+// implementation of the same steps gives the same bits.
+__device__ __forceinline__ float exp_sd(float s) {
+  if (!(s >= -87.0f)) return 0.0f;
+  const float n = rintf(__fmul_rn(s, (float)1.4426950408889634));
+  const float r = __fsub_rn(__fsub_rn(s, __fmul_rn(n, 0.693145751953125f)), __fmul_rn(n, (float)(0.6931471805599453 - 0.693145751953125)));
+  float p = (float)(1.0 / 5040.0);        // 1/7!
+  p = __fadd_rn(__fmul_rn(p, r), (float)(1.0 / 720.0));  // 1/6!
+  p = __fadd_rn(__fmul_rn(p, r), (float)(1.0 / 120.0));  // 1/5!
+  p = __fadd_rn(__fmul_rn(p, r), (float)(1.0 / 24.0));  // 1/4!
+  p = __fadd_rn(__fmul_rn(p, r), (float)(1.0 / 6.0));  // 1/3!
+  p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  const float scale = __int_as_float(((int)n + 127) << 23);
+  return __fmul_rn(p, scale);
+}
+
+// floor(w * 2^24) for 0 <= w <= 1, exactly, from the fp32 bits
+__device__ __forceinline__ uint32_t fixed24(float w) {
+  const uint32_t b = __float_as_uint(w);
+  if (b == 0) return 0;
+  const int sh = (int)((b >> 23) & 0xFF) - 127 + 1;   // W = mant * 2^(e - 23 + 24)
+  const uint32_t mant = (b & 0x7FFFFFu) | 0x800000u;
+  if (sh >= 0) return mant << sh;
+  return sh <= -24 ? 0u : (mant >> (-sh));
+}
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11)
+__device__ __forceinline__ void philox4x32_10(uint32_t c[4], uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c[0], hi0 = __umulhi(0xD2511F53u, c[0]);
+    const uint32_t lo1 = 0xCD9E8D57u * c[2], hi1 = __umulhi(0xCD9E8D57u, c[2]);
+    const uint32_t n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
+    c[0] = n0;
+    c[1] = lo1;
+    c[2] = n2;
+    c[3] = lo0;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+}
+
+// ---- block-wide reductions (1024 threads) -----------------------------------------
+constexpr int ACC_THREADS = 1024;
+constexpr int ACC_EPT = 32;   // logits per thread in the nucleus kernel (vocab <= 32768)
+
+__device__ __forceinline__ uint64_t block_sum_u64(uint64_t v, uint64_t* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  uint64_t t = (l < (int)(blockDim.x >> 5)) ? red[l] : 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  return t;
+}
+
+__device__ __forceinline__ float block_max_f(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = (l < (int)(blockDim.x >> 5)) ? red[l] : -INFINITY;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t = fmaxf(t, __shfl_xor_sync(0xffffffffu, t, o));
+  return t;
+}
+
+// exclusive prefix sum over threads (in thread order) of v; returns this thread's offset
+__device__ __forceinline__ uint64_t block_exscan_u64(uint64_t v, uint64_t* red) {
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  uint64_t x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint64_t y = __shfl_up_sync(0xffffffffu, x, o);
+    if (l >= o) x += y;
+  }
+  __syncthreads();
+  if (l == 31) red[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    uint64_t t = (l < (int)(blockDim.x >> 5)) ? red[l] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint64_t y = __shfl_up_sync(0xffffffffu, t, o);
+      if (l >= o) t += y;
+    }
+    red[l] = t;   // inclusive prefix of warp sums
+  }
+  __syncthreads();
+  return (w > 0 ? red[w - 1] : 0) + x - v;
+}
+
+// ---- greedy: argmax with the lowest id on ties, NaN as -inf ----------------------------
+__device__ int row_argmax(const float* row, int V, uint32_t* err, float* redf, int* redi) {
+  float best = -INFINITY;
+  int bi = 0x7FFFFFFF;
+  bool nan = false;
+  for (int i = threadIdx.x; i < V; i += blockDim.x) {
+    float x = __ldcg(row + i);
+    if (x != x) {
+      nan = true;
+      x = -INFINITY;
+    }
+    if (x > best || (x == best && i < bi)) {
+      best = x;
+      bi = i;
+    }
+  }
+  if (nan) set_error(err, ERR_NAN_LOGITS);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ob > best || (ob == best && oi < bi)) {
+      best = ob;
+      bi = oi;
+    }
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) {
+    redf[w] = best;
+    redi[w] = bi;
+  }
+  __syncthreads();
+  if (w == 0) {
+    const int nw = blockDim.x >> 5;
+    best = l < nw ? redf[l] : -INFINITY;
+    bi = l < nw ? redi[l] : 0x7FFFFFFF;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ob > best || (ob == best && oi < bi)) {
+        best = ob;
+        bi = oi;
+      }
+    }
+    if (l == 0) redi[0] = (bi == 0x7FFFFFFF) ? 0 : bi;
+  }
+  __syncthreads();
+  return redi[0];
+}
+
+// ---- nucleus: the fixed-point top-k / top-p sampler ------------------------------------
+// Thread t owns ids [32t, 32t+32) (ascending id order is thread order, then
+// slot) and keeps their weights W (uint32, <= 2^24) in registers.  Selections
+// are predicates on (W, id); per-thread sums fit 32 bits, block sums 64.
+struct Cut {
+  uint32_t xk;  // top-k: candidates are W > xk, or W == xk and id <= idk
+  int idk;
+  uint32_t xp;  // top-p: kept candidates are W > xp, or W == xp and id <= idp
+  int idp;
+};
+enum Pred : int {
+  P_GE = 1,         // W >= x
+  P_GT = 2,         // W > x
+  P_EQ = 3,         // W == x
+  P_CAND = 4,       // candidate
+  P_CAND_GE = 5,    // candidate and W >= x
+  P_CAND_GT = 6,    // candidate and W > x
+  P_CAND_EQ = 7,    // candidate and W == x
+  P_KEPT = 8,       // kept
+};
+
+template <int P>
+__device__ __forceinline__ bool pred(uint32_t W, int id, const Cut& c, uint32_t x) {
+  const bool cand = W > c.xk || (W == c.xk && id <= c.idk);
+  switch (P) {
+    case P_GE: return W >= x;
+    case P_GT: return W > x;
+    case P_EQ: return W == x;
+    case P_CAND: return cand;
+    case P_CAND_GE: return cand && W >= x;
+    case P_CAND_GT: return cand && W > x;
+    case P_CAND_EQ: return cand && W == x;
+    default: return cand && (W > c.xp || (W == c.xp && id <= c.idp));
+  }
+}
+
+// per-thread sum of W (COUNT: number of ids) over the owned ids selected by P
+template <int P, bool COUNT>
+__device__ __forceinline__ uint32_t lsum(const uint32_t (&W)[ACC_EPT], int base, const Cut& c, uint32_t x) {
+  uint32_t s = 0;
+#pragma unroll
+  for (int e = 0; e < ACC_EPT; ++e)
+    if (pred<P>(W[e], base + e, c, x)) s += COUNT ? 1u : W[e];
+  return s;
+}
+
+// largest x in [0, 2^24] whose block total of lsum<P, COUNT>(x) is >= need (monotone in x)
+template <int P, bool COUNT>
+__device__ __forceinline__ uint32_t search_threshold(const uint32_t (&W)[ACC_EPT], int base, const Cut& c,
+                                                     uint64_t need, uint64_t* red) {
+  uint32_t lo = 0, hi = 1u << 24;
+  while (lo < hi) {
+    const uint32_t mid = lo + (hi - lo + 1) / 2;
+    if (block_sum_u64(lsum<P, COUNT>(W, base, c, mid), red) >= need) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// the n-th (n >= 1) smallest id selected by P, or INT_MAX if there are fewer
+template <int P>
+__device__ __forceinline__ int nth_id(const uint32_t (&W)[ACC_EPT], int base, const Cut& c, uint32_t x,
+                                      uint64_t n, uint64_t* red, int* redi) {
+  const uint64_t mine = lsum<P, true>(W, base, c, x);
+  const uint64_t before = block_exscan_u64(mine, red);
+  if (threadIdx.x == 0) redi[0] = 0x7FFFFFFF;
+  __syncthreads();
+  if (before < n && before + mine >= n) {
+    uint64_t k = before;
+    int hit = 0x7FFFFFFF;
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e)
+      if (pred<P>(W[e], base + e, c, x) && ++k == n) hit = base + e;
+    redi[0] = hit;
+  }
+  __syncthreads();
+  const int out = redi[0];
+  __syncthreads();
+  return out;
+}
+
+__device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* row, int position, int seq,
+                                           float* redf, uint64_t* red, int* redi) {
+  const int V = p.V;
+  const int base = threadIdx.x * ACC_EPT;
+  uint32_t W[ACC_EPT];
+  float mx = -INFINITY;
+  bool nan = false;
+  {
+    // 1. logits (NaN -> -inf; ids >= V are -inf, hence W = 0) and the row maximum
+    float l[ACC_EPT];
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; e += 4) {
+      float4 v = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+      if (base + e + 3 < V) {
+        v = __ldcg(reinterpret_cast<const float4*>(row + base + e));
+      } else {
+        if (base + e < V) v.x = __ldcg(row + base + e);
+        if (base + e + 1 < V) v.y = __ldcg(row + base + e + 1);
+        if (base + e + 2 < V) v.z = __ldcg(row + base + e + 2);
+      }
+      l[e] = v.x; l[e + 1] = v.y; l[e + 2] = v.z; l[e + 3] = v.w;
+    }
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e) {
+      if (l[e] != l[e]) {
+        nan = true;
+        l[e] = -INFINITY;
+      }
+      mx = fmaxf(mx, l[e]);
+    }
+    if (nan) set_error(p.err, ERR_NAN_LOGITS);
+    mx = block_max_f(mx, redf);
+    // 2-3. W_i = floor(exp((l_i - max) / T) * 2^24)
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e) W[e] = fixed24(exp_sd(__fdiv_rn(__fsub_rn(l[e], mx), p.temperature)));
+  }
+  Cut c;
+  c.xk = 0;
+  c.idk = 0x7FFFFFFF;
+  c.xp = 0;
+  c.idp = 0x7FFFFFFF;
+  // 4. top-k candidates
+  if (p.top_k > 0 && p.top_k < V) {
+    c.xk = search_threshold<P_GE, true>(W, base, c, (uint64_t)p.top_k, red);
+    const uint64_t above = block_sum_u64(lsum<P_GT, true>(W, base, c, c.xk), red);
+    c.idk = nth_id<P_EQ>(W, base, c, c.xk, (uint64_t)p.top_k - above, red, redi);
+  }
+  // 5. top-p over the candidates: thr = ceil(P * S / 2^24), P <= 2^24, S < 2^40
+  const uint64_t S = block_sum_u64(lsum<P_CAND, false>(W, base, c, 0), red);
+  if (S == 0) return nth_id<P_CAND>(W, base, c, 0, 1, red, redi);   // all-NaN row: lowest candidate
+  const uint64_t prod = (uint64_t)p.p_fixed * S;
+  const uint64_t thr = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
+  c.xp = search_threshold<P_CAND_GE, false>(W, base, c, thr, red);
+  const uint64_t above = block_sum_u64(lsum<P_CAND_GT, false>(W, base, c, c.xp), red);
+  const uint64_t n_above = block_sum_u64(lsum<P_CAND_GT, true>(W, base, c, c.xp), red);
+  uint64_t ties = thr > above ? (thr - above + c.xp - 1) / c.xp : 0;
+  if (n_above == 0 && ties == 0) ties = 1;
+  c.idp = ties == 0 ? -1 : nth_id<P_CAND_EQ>(W, base, c, c.xp, ties, red, redi);
+  const uint64_t Sk = block_sum_u64(lsum<P_KEPT, false>(W, base, c, 0), red);
+  // 6. the 64-bit draw keyed by (produced position, sequence)
+  uint32_t ctr[4] = {(uint32_t)position, (uint32_t)seq, 0u, 0u};
+  philox4x32_10(ctr, (uint32_t)(p.seed & 0xFFFFFFFFull), (uint32_t)(p.seed >> 32));
+  const uint64_t rnd = ((uint64_t)ctr[0] << 32) | ctr[1];
+  const uint64_t tau = __umul64hi(rnd, Sk);
+  // 7. the first kept id (ascending) whose inclusive cumulative weight exceeds tau
+  const uint64_t mine = lsum<P_KEPT, false>(W, base, c, 0);
+  const uint64_t before = block_exscan_u64(mine, red);
+  if (threadIdx.x == 0) redi[0] = 0x7FFFFFFF;
+  __syncthreads();
+  if (before <= tau && before + mine > tau) {
+    uint64_t cum = before;
+    int pick = 0x7FFFFFFF;
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e) {
+      if (pred<P_KEPT>(W[e], base + e, c, 0)) {
+        cum += W[e];
+        if (cum > tau && pick == 0x7FFFFFFF) pick = base + e;
+      }
+    }
+    redi[0] = pick;
+  }
+  __syncthreads();
+  const int out = redi[0];
+  __syncthreads();
+  return out;
+}
+
+__global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams p) {
+  __shared__ float redf[32];
+  __shared__ uint64_t red[32];
+  __shared__ int redi[32];
+  __shared__ int s_last;
+  pdl_wait();
+  pdl_trigger();
+  const int j = blockIdx.x, sl = blockIdx.y, s = p.seq0 + sl;
+  const float* row = p.logits + (size_t)(sl * p.q + j) * p.V;
+  int t;
+  if (p.temperature <= 0.f) {
+    t = row_argmax(row, p.V, p.err, redf, redi);
+  } else {
+    const int position = __ldcg(p.len + s) + j + 1;   // the produced token's position
+    t = row_nucleus(p, row, position, s, redf, red, redi);
+  }
+  if (threadIdx.x == 0) p.targets[sl * p.q + j] = t;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(p.counters + sl, 1) == p.q - 1);
+  __syncthreads();
+  if (!s_last || threadIdx.x != 0) return;
+  __threadfence();
+  int tg[SDSAT_ATT_MAXQ];
+  for (int i = 0; i < p.q; ++i) tg[i] = __ldcg(p.targets + sl * p.q + i);
+  int m = 0;
+  for (int i = 1; i <= p.n_verify; ++i) {          // Eq. 3: prefix of matching drafts
+    if (__ldcg(p.drafts + sl * p.q + i) != tg[i - 1]) break;
+    m = i;
+  }
+  for (int i = 0; i < p.q; ++i) p.out_tokens[sl * p.q + i] = tg[i];
+  p.accepted_len[sl] = 1 + m;
+  if (p.commit) {
+    const int nl = __ldcg(p.len + s) + 1 + m;
+    if (nl <= p.cap) p.len[s] = nl;
+    else set_error(p.err, ERR_CAPACITY);
+  }
+  p.counters[sl] = 0;
+}
+
+static cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, cudaStream_t st, bool pdl, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.stream = st;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cfg;
+}
+
+cudaError_t launch_accept(const AcceptParams& p, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(p.q, p.nb), dim3(ACC_THREADS), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, accept_kernel, p);
+}
+
+// ---- embedding gather: h[m][:] = E[token[m]][:] (fp32) ---------------------------------
+__global__ void embed_kernel(const int* tokens, const __nv_bfloat16* E, int V, int d, float* h, uint32_t* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int m = blockIdx.x;
+  int t = __ldcg(tokens + m);
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0) set_error(err, ERR_TOKEN);
+    t = 0;
+  }
+  const __nv_bfloat162* src = reinterpret_cast<const __nv_bfloat162*>(E + (size_t)t * d);
+  float2* dst = reinterpret_cast<float2*>(h + (size_t)m * d);
+  for (int i = threadIdx.x; i < d / 2; i += blockDim.x) dst[i] = __bfloat1622float2(src[i]);
+}
+
+cudaError_t launch_embed(const int* tokens, const __nv_bfloat16* E, int V, int d, int M, float* h,
+                         uint32_t* err, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(M), dim3(256), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, embed_kernel, tokens, E, V, d, h, err);
+}
+
+// ---- block input of draft step 1 (mode 1) and draft step 2 (mode 2) --------------------
+__global__ void build_block_kernel(int mode, const int* prev_out, const int* prev_acc, const int* table,
+                                   int table_stride, const int* len, const int* adaptive, int q, int* tokens) {
+  pdl_wait();
+  pdl_trigger();
+  const int sl = blockIdx.x, j = threadIdx.x;
+  if (j >= q) return;
+  int t;
+  if (mode == 1) {
+    t = (j == 0) ? __ldcg(prev_out + sl * q + __ldcg(prev_acc + sl) - 1) : adaptive[j - 1];
+  } else {
+    if (j == 0) t = __ldcg(prev_out + sl * q);
+    else if (table) t = __ldcg(table + (size_t)sl * table_stride + __ldcg(len + sl) + j);
+    else t = __ldcg(prev_out + sl * q + j);
+  }
+  tokens[sl * q + j] = t;
+}
+
+cudaError_t launch_build_block(int mode, const int* prev_out, const int* prev_acc, const int* table,
+                               int table_stride, const int* len, const int* adaptive, int nb, int q,
+                               int* tokens_out, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(nb), dim3(32), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, build_block_kernel, mode, prev_out, prev_acc, table, table_stride, len,
+                            adaptive, q, tokens_out);
+}
+
+// ---- explicit commit / rollback, and prefill commit --------------------------------------
+__global__ void commit_kernel(int* len, const int* new_len, int nb, int cap, uint32_t* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int s = threadIdx.x;
+  if (s >= nb) return;
+  int v = __ldcg(new_len + s);
+  if (v < 0 || v > cap) {
+    set_error(err, ERR_CAPACITY);
+    v = v < 0 ? 0 : cap;
+  }
+  len[s] = v;
+}
+
+cudaError_t launch_commit(int* len, const int* new_len, int nb, int cap, uint32_t* err, cudaStream_t st,
+                          bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(64), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, commit_kernel, len, new_len, nb, cap, err);
+}
+
+__global__ void add_len_kernel(int* len, int seq, int n, int cap, uint32_t* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int v = __ldcg(len + seq) + n;
+  if (v > cap) set_error(err, ERR_CAPACITY);
+  len[seq] = v > cap ? cap : v;
+}
+
+cudaError_t launch_add_len(int* len, int seq, int n, int cap, uint32_t* err, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(1), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, add_len_kernel, len, seq, n, cap, err);
+}
+
+__global__ void exp_kernel(const float* in, float* out, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) out[i] = exp_sd(in[i]);
+}
+
+cudaError_t launch_exp(const float* in, float* out, int n, cudaStream_t st) {
+  exp_kernel<<<(n + 255) / 256, 256, 0, st>>>(in, out, n);
+  return cudaGetLastError();
+}
+
+}  // namespace sdsat

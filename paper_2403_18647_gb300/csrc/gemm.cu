@@ -1,0 +1,417 @@
+// Skinny-M weight-streaming GEMM on the 5th-generation tensor cores.
+//
+// Every projection of the block forward (QKV, O, gate/up, down, LM head) is
+// Y[M, N] = X[M, K] W[N, K]^T with M = b*q <= 64 rows and a weight matrix of
+// 30-330 MB.  The weights are read once per step, so the kernel is bound by
+// HBM bandwidth (decoding is memory-bandwidth bound, Sec. 1; the loop time is
+// almost flat in k, Sec. 3.4.1).  Design:
+//
+//  * Persistent grid of P CTAs; the (128-row tile, 64-wide K chunk) work units
+//    are split evenly in one flat range ("stream-K"), so every CTA streams the
+//    same number of 16 KB weight chunks.  A tile cut between CTAs is reduced
+//    by its last finisher (per-tile counter), summing the partials in CTA
+//    order: deterministic, no spin-wait.
+//  * Warp 0 streams weight chunks with TMA (128-byte swizzle, L2 evict-first)
+//    into a ring of shared-memory stages; it needs nothing from the previous
+//    kernel, so with programmatic dependent launch it starts prefetching while
+//    the previous kernel drains.
+//  * Warps 2-3 build the activation operand per chunk: fp32 rows (optionally
+//    RMS-normalised with the gain, fusing the RMSNorm) split into bf16 hi + lo
+//    parts so that the tensor-core product keeps ~16 mantissa bits of X.
+//  * Warp 1 (one thread) issues tcgen05.mma: D[128 x MPAD] (fp32, TMEM) +=
+//    Wtile[128 x 16] * Xhi^T + Wtile * Xlo^T, four K-steps per chunk.  Two TMEM
+//    accumulators alternate so a tile's epilogue overlaps the next tile's MMAs.
+//  * Warps 4-7 read the accumulator (tcgen05.ld) and run the fused epilogue:
+//    plain store, residual add, RoPE + KV-cache append, or SiLU(gate) * up.
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sdsat {
+
+template <int MPAD>
+struct GemmCfg {
+  static constexpr int STAGES = MPAD <= 16 ? 5 : (MPAD <= 32 ? 4 : 3);
+  static constexpr int W_BYTES = 128 * 128;      // 128 rows x 64 bf16
+  static constexpr int X_BYTES = MPAD * 128;     // MPAD rows x 64 bf16 (hi or lo)
+  static constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
+  static constexpr int STAGING = 128 * (MPAD + 1);
+  static constexpr int TMEM_COLS = 2 * MPAD < 32 ? 32 : 2 * MPAD;
+  static constexpr int NBAR = 3 * STAGES + 5;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 64 * 4 + NBAR * 8 + 32;
+};
+
+__device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
+  return ((g + 1) * P - 1) / T;
+}
+
+// (tensor map, first row) of half h (0: tile rows 0-63, 1: rows 64-127) of tile t
+__device__ __forceinline__ void tile_half_src(const GemmParams& p, int t, int h, int& map, int& row) {
+  if (p.map_mode == MAP_GATEUP) {
+    map = h;
+    row = 64 * t;
+  } else if (p.map_mode == MAP_QKV3) {
+    const int g = 128 * t;
+    map = g / p.rows_per_map;
+    row = g % p.rows_per_map + 64 * h;
+  } else {
+    map = 0;
+    row = 128 * t + 64 * h;
+  }
+}
+
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
+  }
+  return true;
+}
+
+template <int MPAD>
+__device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
+                                               float* staging) {
+  const int M = p.M;
+  if (p.epi == EPI_STORE || p.epi == EPI_RESID) {
+    const int n = 128 * tile + r;
+    if (n < p.N) {
+#pragma unroll
+      for (int m = 0; m < MPAD; ++m) {
+        if (m < M) {
+          float* o = p.out + (size_t)m * p.out_ld + n;
+          *o = (p.epi == EPI_RESID) ? __ldcg(o) + acc[m] : acc[m];
+        }
+      }
+    }
+    return;
+  }
+  // epilogues that combine two TMEM lanes of the tile: exchange through shared memory
+#pragma unroll
+  for (int m = 0; m < MPAD; ++m) staging[r * (MPAD + 1) + m] = acc[m];
+  named_bar_sync(1, 128);
+  if (p.epi == EPI_SWIGLU) {
+    const int j = 64 * tile + r;
+    if (r < 64 && j < p.N) {
+#pragma unroll
+      for (int m = 0; m < MPAD; ++m) {
+        if (m >= M) break;
+        const float g = acc[m];
+        const float u = staging[(r + 64) * (MPAD + 1) + m];
+        p.out[(size_t)m * p.out_ld + j] = g / (1.0f + expf(-g)) * u;
+      }
+    }
+  } else {  // EPI_QKV
+    const int R = p.rows_per_map;
+    const int gf = 128 * tile + r;
+    const int which = gf / R;
+    const int f = gf % R;
+    const int hd = p.hd, half = hd >> 1;
+    const int head = f / hd, i = f % hd;
+    const int partner = (i < half) ? r + half : r - half;
+#pragma unroll
+    for (int m = 0; m < MPAD; ++m) {
+      if (m >= M) break;
+      const int sl = m / p.q, j = m % p.q, s = p.seq0 + sl;
+      const int slot = __ldcg(p.len + s) + j;
+      const float x = acc[m];
+      float val = x;
+      if (which < 2) {
+        int pos = p.positions ? __ldcg(p.positions + m) : slot;
+        if (pos < 0 || pos >= p.rope_len) {
+          set_error(p.err, ERR_POSITION);
+          pos = pos < 0 ? 0 : p.rope_len - 1;
+        }
+        const float y = staging[partner * (MPAD + 1) + m];
+        const float2 cs = p.rope[(size_t)pos * half + (i % half)];
+        val = (i < half) ? x * cs.x - y * cs.y : x * cs.x + y * cs.y;
+      }
+      if (which == 0) {
+        p.out[(size_t)m * p.out_ld + f] = val;
+      } else if (slot < p.cap) {
+        __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
+        cache[(((size_t)s * p.H + head) * p.cap + slot) * hd + i] = __float2bfloat16_rn(val);
+      } else if (i == 0 && which == 1) {
+        set_error(p.err, ERR_CAPACITY);
+      }
+    }
+  }
+  named_bar_sync(1, 128);
+}
+
+template <int MPAD>
+__global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ GemmParams p) {
+  using C = GemmCfg<MPAD>;
+  constexpr int S = C::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* stages = smem;
+  float* staging = reinterpret_cast<float*>(smem + (size_t)S * C::STAGE_BYTES);
+  float* inv_rms = staging + C::STAGING;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(inv_rms + 64);
+  uint64_t* full = bars;             // weights landed (TMA)
+  uint64_t* xfull = bars + S;        // activation operand written
+  uint64_t* empty = bars + 2 * S;    // stage consumed by the tensor core
+  uint64_t* acc_full = bars + 3 * S; // [2] accumulator ready
+  uint64_t* acc_empty = acc_full + 2;// [2] accumulator drained
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* s_last = reinterpret_cast<int*>(tmem_slot + 2);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cta = blockIdx.x;
+  const long long T = (long long)p.n_tiles * p.kc;
+  const long long g0 = (long long)cta * T / p.P, g1 = (long long)(cta + 1) * T / p.P;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&xfull[s], 2);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+
+  if (warp == 0) {
+    // ------------------------------------------------ weight stream (TMA)
+    if (lane == 0) {
+      const int nmaps = p.map_mode == MAP_QKV3 ? 3 : (p.map_mode == MAP_GATEUP ? 2 : 1);
+      for (int i = 0; i < nmaps; ++i) tma_prefetch_desc(&p.tmap[i]);
+      const uint64_t pol = l2_policy_evict_first();
+      int it = 0;
+      for (long long g = g0; g < g1; ++g, ++it) {
+        const int s = it % S;
+        const uint32_t ph = (it / S) & 1;
+        if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, p.err)) break;
+        const int tile = (int)(g / p.kc), kc = (int)(g % p.kc);
+        uint8_t* dst = stages + (size_t)s * C::STAGE_BYTES;
+        mbar_arrive_expect_tx(&full[s], C::W_BYTES);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          int map, row;
+          tile_half_src(p, tile, h, map, row);
+          tma_load_2d(dst + h * 8192, &p.tmap[map], &full[s], kc * 64, row, pol);
+        }
+      }
+      if (*abort_flag) {  // let every copy in flight land before the CTA exits
+        for (int i = std::max(0, it - S); i < it; ++i) mbar_wait_drain(&full[i % S], (i / S) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ tensor-core issue
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(128, MPAD);
+      int it = 0, seg = 0;
+      long long g = g0;
+      bool ok = true;
+      while (ok && g < g1) {
+        const int tile = (int)(g / p.kc);
+        const long long gend = std::min(g1, (long long)(tile + 1) * p.kc);
+        const int buf = seg & 1;
+        if (!mbar_wait_bounded(&acc_empty[buf], ((seg >> 1) & 1) ^ 1, abort_flag, p.err)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + buf * MPAD;
+        const long long gstart = g;
+        for (; g < gend; ++g, ++it) {
+          const int s = it % S;
+          const uint32_t ph = (it / S) & 1;
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag, p.err) ||
+              !mbar_wait_bounded(&xfull[s], ph, abort_flag, p.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t wa = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
+          const uint32_t xh = wa + C::W_BYTES, xl = xh + C::X_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = sdesc_sw128(wa + kk * 32);
+            umma_bf16(d, ad, sdesc_sw128(xh + kk * 32), idesc, (g != gstart || kk > 0) ? 1u : 0u);
+            umma_bf16(d, ad, sdesc_sw128(xl + kk * 32), idesc, 1u);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(&acc_full[buf]);
+        ++seg;
+      }
+      if (*abort_flag) {  // wait for issued MMAs before shared memory goes away
+        umma_commit(drain);
+        mbar_wait_drain(drain, 0);
+      }
+    }
+  } else if (warp < 4) {
+    // ------------------------------------------------ activation operand (hi/lo bf16)
+    const int tid = threadIdx.x - 64;
+    pdl_wait();
+    if (p.norm) {
+      for (int m = warp - 2; m < p.M; m += 2) {
+        const float* xr = p.x + (size_t)m * p.x_ld;
+        float ss = 0.f;
+        for (int k = lane * 4; k < p.K; k += 128) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + k));
+          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        if (lane == 0) inv_rms[m] = 1.0f / sqrtf(ss / (float)p.K + p.eps);
+      }
+      named_bar_sync(2, 64);
+    }
+    int it = 0;
+    for (long long g = g0; g < g1; ++g, ++it) {
+      const int s = it % S;
+      const uint32_t ph = (it / S) & 1;
+      if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, p.err)) break;
+      const int k0 = (int)(g % p.kc) * 64;
+      uint8_t* xh = stages + (size_t)s * C::STAGE_BYTES + C::W_BYTES;
+      uint8_t* xl = xh + C::X_BYTES;
+      for (int gr = tid; gr < MPAD * 8; gr += 64) {
+        const int m = gr >> 3, c = gr & 7, k = k0 + c * 8;
+        float v[8];
+        if (m < p.M && k < p.K) {
+          const float4* src = reinterpret_cast<const float4*>(p.x + (size_t)m * p.x_ld + k);
+          const float4 a = __ldcg(src), b = __ldcg(src + 1);
+          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+          if (p.norm) {
+            const float sc = inv_rms[m];
+            const uint4 graw = *reinterpret_cast<const uint4*>(p.gain + k);
+            const __nv_bfloat16* gg = reinterpret_cast<const __nv_bfloat16*>(&graw);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = v[e] * sc * __bfloat162float(gg[e]);
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) v[e] = 0.f;
+        }
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]), h1 = __float2bfloat16_rn(v[2 * e + 1]);
+          const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * e] - __bfloat162float(h0));
+          const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1));
+          hi[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+          lo[e] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+        }
+        const int off = m * 128 + ((c ^ (m & 7)) << 4);
+        *reinterpret_cast<uint4*>(xh + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(xl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&xfull[s]);
+    }
+  } else {
+    // ------------------------------------------------ epilogue (TMEM -> registers -> global)
+    const int e = warp & 3;   // TMEM lane quarter this warp may access
+    const int r = e * 32 + lane;
+    pdl_wait();
+    int seg = 0;
+    long long g = g0;
+    while (g < g1) {
+      const int tile = (int)(g / p.kc);
+      g = std::min(g1, (long long)(tile + 1) * p.kc);
+      const int buf = seg & 1;
+      if (!mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err)) break;
+      tc_fence_after();
+      float acc[MPAD];
+#pragma unroll
+      for (int c = 0; c < MPAD; c += 16)
+        tmem_ld16(tmem + ((uint32_t)(e * 32) << 16) + buf * MPAD + c, acc + c);
+      tmem_wait_ld();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      ++seg;
+
+      const long long tstart = (long long)tile * p.kc;
+      const int c_lo = (int)cta_of_chunk(tstart, T, p.P);
+      const int c_hi = (int)cta_of_chunk(tstart + p.kc - 1, T, p.P);
+      if (c_hi > c_lo) {
+        // this tile is shared: publish the partial, the last contributor reduces
+        const int my_first_tile = (int)(g0 / p.kc);
+        const int slot = (tile == my_first_tile) ? 0 : 1;
+        float* mine = p.partials + (size_t)(cta * 2 + slot) * MPAD * 128;
+#pragma unroll
+        for (int m = 0; m < MPAD; ++m)
+          if (m < p.M) mine[m * 128 + r] = acc[m];
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (r == 0) *s_last = (atomicAdd(&p.counters[tile], 1) == c_hi - c_lo);
+        named_bar_sync(1, 128);
+        if (!*s_last) continue;
+        __threadfence();
+#pragma unroll
+        for (int m = 0; m < MPAD; ++m) acc[m] = 0.f;
+        for (int j = c_lo; j <= c_hi; ++j) {
+          const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
+          const float* src = p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128;
+#pragma unroll
+          for (int m = 0; m < MPAD; ++m)
+            if (m < p.M) acc[m] += __ldcg(src + m * 128 + r);
+        }
+        if (r == 0) p.counters[tile] = 0;
+      }
+      epilogue_final<MPAD>(p, tile, r, acc, staging);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+int gemm_mpad(int M) { return M <= 16 ? 16 : (M <= 32 ? 32 : 64); }
+
+size_t gemm_smem_bytes(int mpad) {
+  return mpad == 16 ? GemmCfg<16>::SMEM : (mpad == 32 ? GemmCfg<32>::SMEM : GemmCfg<64>::SMEM);
+}
+
+cudaError_t gemm_prepare() {
+  cudaError_t e = cudaFuncSetAttribute(gemm_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)GemmCfg<16>::SMEM);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(gemm_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)GemmCfg<32>::SMEM);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemm_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)GemmCfg<64>::SMEM);
+}
+
+cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl) {
+  const long long T = (long long)p.n_tiles * p.kc;
+  p.P = (int)std::min<long long>(num_sms, T);
+  const int mpad = gemm_mpad(p.M);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.P);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = gemm_smem_bytes(mpad);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (mpad == 16) return cudaLaunchKernelEx(&cfg, gemm_kernel<16>, p);
+  if (mpad == 32) return cudaLaunchKernelEx(&cfg, gemm_kernel<32>, p);
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<64>, p);
+}
+
+}  // namespace sdsat

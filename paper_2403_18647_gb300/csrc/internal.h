@@ -1,0 +1,116 @@
+// Internal declarations shared by the libsdsat translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace sdsat {
+
+// ---- skinny weight-streaming GEMM --------------------------------------------
+// Tiles of 128 output features x 64 K-elements; the 128 rows come from two
+// 64-row TMA boxes ("halves") whose source depends on the map mode.
+enum GemmMap : int {
+  MAP_PLAIN = 0,    // one matrix [N][K]: tile t = rows 128t .. 128t+127
+  MAP_QKV3 = 1,     // three matrices of rows_per_map rows each (q, k, v), stacked
+  MAP_GATEUP = 2,   // two matrices [F][K]: tile t = gate rows 64t.. and up rows 64t..
+};
+enum GemmEpi : int {
+  EPI_STORE = 0,    // out[m][n] = acc
+  EPI_RESID = 1,    // out[m][n] += acc (residual stream)
+  EPI_QKV = 2,      // RoPE on q, k; q -> out (fp32), k, v -> KV cache (bf16)
+  EPI_SWIGLU = 3,   // out[m][j] = silu(gate) * up
+};
+
+struct GemmParams {
+  CUtensorMap tmap[3];
+  int map_mode;
+  int N;              // output features (MAP_GATEUP: F)
+  int K;
+  int rows_per_map;   // MAP_QKV3: rows of each of q, k, v
+  int n_tiles;
+  int kc;             // K chunks of 64
+  int P;              // CTAs
+  int M;              // activation rows (<= MPAD)
+  // X source: fp32 [M][x_ld]; norm != 0 -> X = x * inv_rms(row) * gain
+  const float* x;
+  int x_ld;
+  int norm;
+  const __nv_bfloat16* gain;
+  float eps;
+  // epilogue
+  int epi;
+  float* out;
+  int out_ld;
+  // EPI_QKV
+  __nv_bfloat16* k_layer;   // KV cache of this layer: [B][H][cap][hd]
+  __nv_bfloat16* v_layer;
+  int H, hd, cap, q, seq0;
+  const int* len;           // committed lengths [B] (device)
+  const int* positions;     // [M] or null
+  const float2* rope;       // [rope_len][hd/2] (cos, sin)
+  int rope_len;
+  // scratch (exclusive to the running GEMM)
+  float* partials;          // [P][2][MPAD][128]
+  int* counters;            // [n_tiles], zero between launches
+  uint32_t* err;
+};
+
+int gemm_mpad(int M);                 // 16, 32 or 64
+size_t gemm_smem_bytes(int mpad);
+cudaError_t gemm_prepare();           // set smem attributes (idempotent)
+cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl);
+
+// ---- attention -------------------------------------------------------------
+constexpr int ATT_CHUNK = 128;
+#define SDSAT_ATT_MAXQ 16
+struct AttnParams {
+  const float* Q;       // [rows][q_ld] (row = sl*q + j), head h at column h*hd
+  int q_ld;
+  const __nv_bfloat16* k;   // [B][H][cap][hd] (this layer)
+  const __nv_bfloat16* v;
+  const int* len;       // [B]
+  int seq0, nb, q, H, hd, cap;
+  float* out;           // [rows][out_ld]
+  int out_ld;
+  float* part_o;        // [rows][H][nch_max][hd]
+  float* part_ml;       // [rows][H][nch_max][2]
+  int nch_max;
+  int* counters;        // [nb][H]
+  uint32_t* err;
+};
+cudaError_t launch_attention(const AttnParams& p, cudaStream_t st, bool pdl);
+
+// ---- embedding, acceptance, block building ------------------------------------
+cudaError_t launch_embed(const int* tokens, const __nv_bfloat16* E, int V, int d, int M, float* h,
+                         uint32_t* err, cudaStream_t st, bool pdl);
+
+struct AcceptParams {
+  const float* logits;      // [nb*q][V]
+  const int* drafts;        // [nb*q]
+  int seq0, nb, q, V, n_verify;
+  float temperature, top_p;
+  uint32_t p_fixed;         // round(top_p * 2^24)
+  uint64_t seed;
+  int top_k;
+  int* len;                 // [B] committed lengths
+  int cap;
+  int commit;
+  int* accepted_len;        // [nb]
+  int* out_tokens;          // [nb*q]
+  int* targets;             // scratch [nb*q]
+  int* counters;            // scratch [nb], zero between launches
+  uint32_t* err;
+};
+cudaError_t launch_accept(const AcceptParams& p, cudaStream_t st, bool pdl);
+
+cudaError_t launch_build_block(int mode, const int* prev_out, const int* prev_acc, const int* table,
+                               int table_stride, const int* len, const int* adaptive, int nb, int q,
+                               int* tokens_out, cudaStream_t st, bool pdl);
+cudaError_t launch_commit(int* len, const int* new_len, int nb, int cap, uint32_t* err, cudaStream_t st,
+                          bool pdl);
+cudaError_t launch_add_len(int* len, int seq, int n, int cap, uint32_t* err, cudaStream_t st, bool pdl);
+cudaError_t launch_exp(const float* in, float* out, int n, cudaStream_t st);
+
+}  // namespace sdsat

@@ -1,0 +1,626 @@
+// libsdsat host side: the C ABI declared in include/sdsat.h.
+//
+// A context holds the borrowed weight pointers, one TMA descriptor per
+// weight matrix, the RoPE table and the workspaces of one block forward; a KV
+// object holds the cache and the device-resident committed lengths.  Every
+// compute entry point only validates arguments and enqueues kernels on the
+// context stream (programmatic dependent launch between consecutive kernels),
+// so the whole decode loop can run, and be graph-captured, without the host.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "../../include/sdsat.h"
+#include "internal.h"
+
+using namespace sdsat;
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encode() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_encode != nullptr;
+}
+
+// bf16 [rows][cols] row-major, boxes of 64 rows x 64 columns, 128-byte swizzle
+bool make_wmap(CUtensorMap* map, const void* ptr, int rows, int cols) {
+  if (!get_encode()) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct LayerMaps {
+  CUtensorMap q, k, v, o, gate, up, down;
+};
+
+constexpr int MAX_GEMM_TILES = 1 << 16;
+
+}  // namespace
+
+struct sdsat_ctx {
+  sdsat_config cfg{};
+  bool has_weights = false;
+  sdsat_weights w{};
+  std::vector<sdsat_layer_weights> layers;
+  std::vector<LayerMaps> maps;
+  CUtensorMap head_map{};
+  cudaStream_t stream = nullptr;
+  int device = 0, num_sms = 0;
+  // workspaces
+  float2* rope = nullptr;
+  float* h = nullptr;
+  float* qbuf = nullptr;
+  float* attn = nullptr;
+  float* act = nullptr;
+  float* partials = nullptr;
+  int* gemm_counters = nullptr;
+  float* att_part_o = nullptr;
+  float* att_part_ml = nullptr;
+  int att_nch = 0;
+  int* att_counters = nullptr;
+  int* acc_targets = nullptr;
+  int* acc_counters = nullptr;
+  int* adaptive = nullptr;
+  uint32_t* err = nullptr;
+  std::vector<void*> allocs;
+};
+
+struct sdsat_kv {
+  sdsat_ctx* ctx = nullptr;
+  int batch = 0, cap = 0;
+  __nv_bfloat16* k = nullptr;
+  __nv_bfloat16* v = nullptr;
+  int* len = nullptr;
+};
+
+namespace {
+
+template <typename T>
+bool dalloc(sdsat_ctx* c, T** p, size_t count) {
+  void* q = nullptr;
+  if (cudaMalloc(&q, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) return false;
+  if (cudaMemset(q, 0, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) {
+    cudaFree(q);
+    return false;
+  }
+  c->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return true;
+}
+
+sdsat_status check_cfg(const sdsat_config& c) {
+  if (c.n_layers < 1 || c.d_model < 8 || c.n_heads < 1 || c.head_dim < 1 || c.ffn_dim < 8 || c.vocab < 2 ||
+      c.max_position < 1 || c.n_adaptive < 1 || c.n_adaptive > SDSAT_MAX_ADAPTIVE || !(c.rms_eps >= 0.f) ||
+      !(c.rope_theta > 0.f))
+    return SDSAT_EINVAL;
+  if (c.d_model % 8 || c.ffn_dim % 8) return SDSAT_EINVAL;
+  if (c.n_kv_heads != c.n_heads) return SDSAT_EUNSUPPORTED;
+  if (c.head_dim != 64 && c.head_dim != 128) return SDSAT_EUNSUPPORTED;
+  if ((c.n_heads * c.head_dim) % 128) return SDSAT_EUNSUPPORTED;
+  for (int i = 0; i < c.n_adaptive; ++i)
+    if (c.adaptive_ids[i] < 0 || c.adaptive_ids[i] >= c.vocab) return SDSAT_EINVAL;
+  return SDSAT_OK;
+}
+
+GemmParams gemm_base(sdsat_ctx* c, int M) {
+  GemmParams g;
+  std::memset(&g, 0, sizeof(g));
+  g.M = M;
+  g.partials = c->partials;
+  g.counters = c->gemm_counters;
+  g.err = c->err;
+  g.eps = c->cfg.rms_eps;
+  return g;
+}
+
+void set_plain(GemmParams& g, const CUtensorMap& m, int N, int K) {
+  g.tmap[0] = m;
+  g.map_mode = MAP_PLAIN;
+  g.N = N;
+  g.K = K;
+  g.n_tiles = (N + 127) / 128;
+  g.kc = (K + 63) / 64;
+}
+
+// one block forward of sequences seq0 .. seq0+nb-1, q rows each
+sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const int32_t* tokens,
+                     const int32_t* positions, float* logits) {
+  const sdsat_config& cf = c->cfg;
+  const int M = nb * q, d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd;
+  cudaStream_t st = c->stream;
+  const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
+  if (launch_embed(tokens, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, d, M, c->h, c->err, st,
+                   true) != cudaSuccess)
+    return SDSAT_ECUDA;
+  for (int l = 0; l < cf.n_layers; ++l) {
+    const sdsat_layer_weights& W = c->layers[l];
+    const LayerMaps& mp = c->maps[l];
+    // QKV projection with the fused RMSNorm, RoPE and KV append
+    GemmParams g = gemm_base(c, M);
+    g.tmap[0] = mp.q;
+    g.tmap[1] = mp.k;
+    g.tmap[2] = mp.v;
+    g.map_mode = MAP_QKV3;
+    g.N = 3 * R;
+    g.K = d;
+    g.rows_per_map = R;
+    g.n_tiles = 3 * R / 128;
+    g.kc = (d + 63) / 64;
+    g.x = c->h;
+    g.x_ld = d;
+    g.norm = 1;
+    g.gain = static_cast<const __nv_bfloat16*>(W.attn_norm);
+    g.epi = EPI_QKV;
+    g.out = c->qbuf;
+    g.out_ld = R;
+    g.k_layer = kv->k + l * layer_elems;
+    g.v_layer = kv->v + l * layer_elems;
+    g.H = H;
+    g.hd = hd;
+    g.cap = kv->cap;
+    g.q = q;
+    g.seq0 = seq0;
+    g.len = kv->len;
+    g.positions = positions;
+    g.rope = c->rope;
+    g.rope_len = cf.max_position;
+    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    // block-causal attention
+    AttnParams a;
+    std::memset(&a, 0, sizeof(a));
+    a.Q = c->qbuf;
+    a.q_ld = R;
+    a.k = kv->k + l * layer_elems;
+    a.v = kv->v + l * layer_elems;
+    a.len = kv->len;
+    a.seq0 = seq0;
+    a.nb = nb;
+    a.q = q;
+    a.H = H;
+    a.hd = hd;
+    a.cap = kv->cap;
+    a.out = c->attn;
+    a.out_ld = R;
+    a.part_o = c->att_part_o;
+    a.part_ml = c->att_part_ml;
+    a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
+    a.counters = c->att_counters;
+    a.err = c->err;
+    if (launch_attention(a, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    // O projection + residual
+    g = gemm_base(c, M);
+    set_plain(g, mp.o, d, R);
+    g.x = c->attn;
+    g.x_ld = R;
+    g.epi = EPI_RESID;
+    g.out = c->h;
+    g.out_ld = d;
+    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    // gate/up with the fused RMSNorm and SiLU(gate) * up
+    g = gemm_base(c, M);
+    g.tmap[0] = mp.gate;
+    g.tmap[1] = mp.up;
+    g.map_mode = MAP_GATEUP;
+    g.N = F;
+    g.K = d;
+    g.n_tiles = (F + 63) / 64;
+    g.kc = (d + 63) / 64;
+    g.x = c->h;
+    g.x_ld = d;
+    g.norm = 1;
+    g.gain = static_cast<const __nv_bfloat16*>(W.ffn_norm);
+    g.epi = EPI_SWIGLU;
+    g.out = c->act;
+    g.out_ld = F;
+    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    // down projection + residual
+    g = gemm_base(c, M);
+    set_plain(g, mp.down, d, F);
+    g.x = c->act;
+    g.x_ld = F;
+    g.epi = EPI_RESID;
+    g.out = c->h;
+    g.out_ld = d;
+    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+  }
+  if (logits) {
+    GemmParams g = gemm_base(c, M);
+    set_plain(g, c->head_map, cf.vocab, d);
+    g.x = c->h;
+    g.x_ld = d;
+    g.norm = 1;
+    g.gain = static_cast<const __nv_bfloat16*>(c->w.final_norm);
+    g.epi = EPI_STORE;
+    g.out = logits;
+    g.out_ld = cf.vocab;
+    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+  }
+  return SDSAT_OK;
+}
+
+sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, const int32_t* drafts, int b, int q,
+                           int n_verify, float top_p, float temperature, uint64_t seed, int top_k, int32_t* acc,
+                           int32_t* out, int commit) {
+  if (!c || !kv || kv->ctx != c || !logits || !drafts || !acc || !out) return SDSAT_EINVAL;
+  if (b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
+  if (n_verify < 0 || n_verify >= q || top_k < 0) return SDSAT_EINVAL;
+  if (temperature > 0.f && !(top_p >= 0.f)) return SDSAT_EINVAL;
+  if (temperature > 0.f && c->cfg.vocab > 32768) return SDSAT_EUNSUPPORTED;
+  AcceptParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.logits = logits;
+  p.drafts = drafts;
+  p.seq0 = 0;
+  p.nb = b;
+  p.q = q;
+  p.V = c->cfg.vocab;
+  p.n_verify = n_verify;
+  p.temperature = temperature;
+  p.top_p = top_p;
+  const double pf = std::nearbyint((double)top_p * 16777216.0);
+  p.p_fixed = (uint32_t)std::min(std::max(pf, 0.0), 16777216.0);
+  p.seed = seed;
+  p.top_k = top_k;
+  p.len = kv->len;
+  p.cap = kv->cap;
+  p.commit = commit;
+  p.accepted_len = acc;
+  p.out_tokens = out;
+  p.targets = c->acc_targets;
+  p.counters = c->acc_counters;
+  p.err = c->err;
+  return launch_accept(p, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* sdsat_status_string(sdsat_status s) {
+  switch (s) {
+    case SDSAT_OK: return "ok";
+    case SDSAT_EINVAL: return "invalid argument";
+    case SDSAT_ENOMEM: return "device allocation failed";
+    case SDSAT_ECAPACITY: return "capacity exceeded";
+    case SDSAT_ECUDA: return "CUDA error";
+    case SDSAT_EDEVICE: return "device-detected error";
+    case SDSAT_EUNSUPPORTED: return "unsupported configuration";
+  }
+  return "unknown status";
+}
+
+void sdsat_destroy(sdsat_ctx* c) {
+  if (!c) return;
+  cudaStreamSynchronize(c->stream);
+  for (void* p : c->allocs) cudaFree(p);
+  delete c;
+}
+
+sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void* stream, sdsat_ctx** out) {
+  if (!cfg || !out) return SDSAT_EINVAL;
+  *out = nullptr;
+  const sdsat_status cs = check_cfg(*cfg);
+  if (cs != SDSAT_OK) return cs;
+  sdsat_ctx* c = new (std::nothrow) sdsat_ctx();
+  if (!c) return SDSAT_ENOMEM;
+  c->cfg = *cfg;
+  c->stream = static_cast<cudaStream_t>(stream);
+  if (cudaGetDevice(&c->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess ||
+      gemm_prepare() != cudaSuccess) {
+    delete c;
+    return SDSAT_ECUDA;
+  }
+  const int L = cfg->n_layers, d = cfg->d_model, R = cfg->n_heads * cfg->head_dim, F = cfg->ffn_dim;
+  if (w) {
+    if (!w->layers || !aligned16(w->embed) || !aligned16(w->final_norm) || !aligned16(w->lm_head)) {
+      delete c;
+      return SDSAT_EINVAL;
+    }
+    c->has_weights = true;
+    c->w = *w;
+    c->layers.assign(w->layers, w->layers + L);
+    c->maps.resize(L);
+    for (int l = 0; l < L; ++l) {
+      const sdsat_layer_weights& W = c->layers[l];
+      if (!aligned16(W.attn_norm) || !aligned16(W.ffn_norm) || !aligned16(W.wq) || !aligned16(W.wk) ||
+          !aligned16(W.wv) || !aligned16(W.wo) || !aligned16(W.w_gate) || !aligned16(W.w_up) ||
+          !aligned16(W.w_down)) {
+        delete c;
+        return SDSAT_EINVAL;
+      }
+      LayerMaps& m = c->maps[l];
+      if (!make_wmap(&m.q, W.wq, R, d) || !make_wmap(&m.k, W.wk, R, d) || !make_wmap(&m.v, W.wv, R, d) ||
+          !make_wmap(&m.o, W.wo, d, R) || !make_wmap(&m.gate, W.w_gate, F, d) || !make_wmap(&m.up, W.w_up, F, d) ||
+          !make_wmap(&m.down, W.w_down, d, F)) {
+        delete c;
+        return SDSAT_ECUDA;
+      }
+    }
+    if (!make_wmap(&c->head_map, w->lm_head, cfg->vocab, d)) {
+      delete c;
+      return SDSAT_ECUDA;
+    }
+  }
+  // RoPE table: angle = pos * theta^(-2i/hd), computed in double
+  const int half = cfg->head_dim / 2;
+  std::vector<float2> rope((size_t)cfg->max_position * half);
+  for (int p = 0; p < cfg->max_position; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double ang = (double)p * std::pow((double)cfg->rope_theta, -2.0 * i / cfg->head_dim);
+      rope[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+    }
+  const int rows = SDSAT_MAX_ROWS;
+  c->att_nch = (cfg->max_position + ATT_CHUNK - 1) / ATT_CHUNK;
+  bool ok = dalloc(c, &c->rope, rope.size()) && dalloc(c, &c->h, (size_t)rows * d) &&
+            dalloc(c, &c->qbuf, (size_t)rows * R) && dalloc(c, &c->attn, (size_t)rows * R) &&
+            dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 64 * 128) &&
+            dalloc(c, &c->gemm_counters, MAX_GEMM_TILES) &&
+            dalloc(c, &c->att_part_o, (size_t)rows * cfg->n_heads * c->att_nch * cfg->head_dim) &&
+            dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * c->att_nch * 2) &&
+            dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
+            dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
+            dalloc(c, &c->err, 1);
+  if (!ok) {
+    sdsat_destroy(c);
+    return SDSAT_ENOMEM;
+  }
+  int ids[SDSAT_MAX_ADAPTIVE];
+  for (int i = 0; i < SDSAT_MAX_ADAPTIVE; ++i)
+    ids[i] = cfg->n_adaptive == 1 ? cfg->adaptive_ids[0] : cfg->adaptive_ids[std::min(i, cfg->n_adaptive - 1)];
+  if (cudaMemcpy(c->rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemcpy(c->adaptive, ids, sizeof(ids), cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaDeviceSynchronize() != cudaSuccess) {
+    sdsat_destroy(c);
+    return SDSAT_ECUDA;
+  }
+  *out = c;
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_set_stream(sdsat_ctx* c, void* stream) {
+  if (!c) return SDSAT_EINVAL;
+  c->stream = static_cast<cudaStream_t>(stream);
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** out) {
+  if (!c || !out || batch < 1 || max_len < 1) return SDSAT_EINVAL;
+  *out = nullptr;
+  if (max_len > c->cfg.max_position) return SDSAT_ECAPACITY;
+  sdsat_kv* kv = new (std::nothrow) sdsat_kv();
+  if (!kv) return SDSAT_ENOMEM;
+  kv->ctx = c;
+  kv->batch = batch;
+  kv->cap = max_len;
+  const size_t n = (size_t)c->cfg.n_layers * batch * c->cfg.n_heads * max_len * c->cfg.head_dim;
+  void *k = nullptr, *v = nullptr, *len = nullptr;
+  if (cudaMalloc(&k, n * 2) != cudaSuccess || cudaMalloc(&v, n * 2) != cudaSuccess ||
+      cudaMalloc(&len, batch * sizeof(int)) != cudaSuccess) {
+    cudaFree(k);
+    cudaFree(v);
+    cudaFree(len);
+    delete kv;
+    return SDSAT_ENOMEM;
+  }
+  if (cudaMemset(k, 0, n * 2) != cudaSuccess || cudaMemset(v, 0, n * 2) != cudaSuccess ||
+      cudaMemset(len, 0, batch * sizeof(int)) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+    cudaFree(k);
+    cudaFree(v);
+    cudaFree(len);
+    delete kv;
+    return SDSAT_ECUDA;
+  }
+  kv->k = static_cast<__nv_bfloat16*>(k);
+  kv->v = static_cast<__nv_bfloat16*>(v);
+  kv->len = static_cast<int*>(len);
+  *out = kv;
+  return SDSAT_OK;
+}
+
+void sdsat_kv_destroy(sdsat_kv* kv) {
+  if (!kv) return;
+  cudaStreamSynchronize(kv->ctx->stream);
+  cudaFree(kv->k);
+  cudaFree(kv->v);
+  cudaFree(kv->len);
+  delete kv;
+}
+
+sdsat_status sdsat_kv_info(const sdsat_kv* kv, void** k_dev, void** v_dev, int32_t** len_dev, int* batch,
+                           int* max_len) {
+  if (!kv) return SDSAT_EINVAL;
+  if (k_dev) *k_dev = kv->k;
+  if (v_dev) *v_dev = kv->v;
+  if (len_dev) *len_dev = kv->len;
+  if (batch) *batch = kv->batch;
+  if (max_len) *max_len = kv->cap;
+  return SDSAT_OK;
+}
+
+static sdsat_status kv_copy(sdsat_ctx* c, const sdsat_kv* kv, int layer, int seq, int slot0, int n, const void* ks,
+                            const void* vs, void* kd, void* vd) {
+  if (!c || !kv || kv->ctx != c || layer < 0 || layer >= c->cfg.n_layers || seq < 0 || seq >= kv->batch ||
+      slot0 < 0 || n < 0 || slot0 + n > kv->cap)
+    return SDSAT_EINVAL;
+  if (n == 0) return SDSAT_OK;
+  const int H = c->cfg.n_heads, hd = c->cfg.head_dim;
+  const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
+  const size_t off = layer * layer_elems + ((size_t)seq * H * kv->cap + slot0) * hd;
+  const size_t cache_pitch = (size_t)kv->cap * hd * 2, buf_pitch = (size_t)n * hd * 2, width = buf_pitch;
+  for (int which = 0; which < 2; ++which) {
+    __nv_bfloat16* cache = (which == 0 ? kv->k : kv->v) + off;
+    cudaError_t e;
+    if (ks || vs) {
+      e = cudaMemcpy2DAsync(cache, cache_pitch, which == 0 ? ks : vs, buf_pitch, width, H, cudaMemcpyDeviceToDevice,
+                            c->stream);
+    } else {
+      e = cudaMemcpy2DAsync(which == 0 ? kd : vd, buf_pitch, cache, cache_pitch, width, H, cudaMemcpyDeviceToDevice,
+                            c->stream);
+    }
+    if (e != cudaSuccess) return SDSAT_ECUDA;
+  }
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_kv_write(sdsat_ctx* c, sdsat_kv* kv, int layer, int seq, int slot0, int n, const void* k_src_dev,
+                            const void* v_src_dev) {
+  if (!k_src_dev || !v_src_dev) return SDSAT_EINVAL;
+  return kv_copy(c, kv, layer, seq, slot0, n, k_src_dev, v_src_dev, nullptr, nullptr);
+}
+
+sdsat_status sdsat_kv_read(sdsat_ctx* c, const sdsat_kv* kv, int layer, int seq, int slot0, int n, void* k_dst_dev,
+                           void* v_dst_dev) {
+  if (!k_dst_dev || !v_dst_dev) return SDSAT_EINVAL;
+  return kv_copy(c, kv, layer, seq, slot0, n, nullptr, nullptr, k_dst_dev, v_dst_dev);
+}
+
+sdsat_status sdsat_block_forward(sdsat_ctx* c, sdsat_kv* kv, const int32_t* tokens_dev,
+                                 const int32_t* positions_dev, int b, int q, float* logits_dev) {
+  if (!c || !kv || kv->ctx != c || !c->has_weights || !tokens_dev || !logits_dev) return SDSAT_EINVAL;
+  if (b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
+  return forward(c, kv, 0, b, q, tokens_dev, positions_dev, logits_dev);
+}
+
+sdsat_status sdsat_prefill(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* tokens_dev, int n) {
+  if (!c || !kv || kv->ctx != c || !c->has_weights || !tokens_dev || seq < 0 || seq >= kv->batch || n < 0)
+    return SDSAT_EINVAL;
+  if (n > kv->cap) return SDSAT_ECAPACITY;
+  for (int i = 0; i < n; i += SDSAT_MAX_Q) {
+    const int qn = std::min(SDSAT_MAX_Q, n - i);
+    const sdsat_status s = forward(c, kv, seq, 1, qn, tokens_dev + i, nullptr, nullptr);
+    if (s != SDSAT_OK) return s;
+    if (launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, true) != cudaSuccess) return SDSAT_ECUDA;
+  }
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_accept_greedy(sdsat_ctx* c, sdsat_kv* kv, const float* logits_dev, const int32_t* drafts_dev,
+                                 int b, int q, int n_verify, int32_t* accepted_len_dev, int32_t* out_tokens_dev,
+                                 int commit) {
+  return accept_common(c, kv, logits_dev, drafts_dev, b, q, n_verify, 1.f, 0.f, 0, 0, accepted_len_dev,
+                       out_tokens_dev, commit);
+}
+
+sdsat_status sdsat_accept_nucleus(sdsat_ctx* c, sdsat_kv* kv, const float* logits_dev, const int32_t* drafts_dev,
+                                  int b, int q, int n_verify, float top_p, float temperature, uint64_t rng_seed,
+                                  int top_k, int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit) {
+  return accept_common(c, kv, logits_dev, drafts_dev, b, q, n_verify, top_p, temperature, rng_seed, top_k,
+                       accepted_len_dev, out_tokens_dev, commit);
+}
+
+sdsat_status sdsat_kv_commit(sdsat_ctx* c, sdsat_kv* kv, const int32_t* new_len_dev, int b) {
+  if (!c || !kv || kv->ctx != c || !new_len_dev || b < 1 || b > kv->batch || b > 64) return SDSAT_EINVAL;
+  return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, true) == cudaSuccess ? SDSAT_OK
+                                                                                                 : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_kv_lengths(sdsat_ctx* c, const sdsat_kv* kv, int32_t* lens_dev, int b) {
+  if (!c || !kv || kv->ctx != c || !lens_dev || b < 1 || b > kv->batch) return SDSAT_EINVAL;
+  return cudaMemcpyAsync(lens_dev, kv->len, b * sizeof(int), cudaMemcpyDeviceToDevice, c->stream) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_build_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32_t* prev_out_dev,
+                               const int32_t* prev_acc_dev, const int32_t* draft_table_dev, int table_stride,
+                               int b, int q, int32_t* tokens_out_dev) {
+  if (!c || !kv || kv->ctx != c || !prev_out_dev || !prev_acc_dev || !tokens_out_dev) return SDSAT_EINVAL;
+  if ((mode != 1 && mode != 2) || b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q) return SDSAT_EINVAL;
+  if (mode == 1 && c->cfg.n_adaptive > 1 && q - 1 > c->cfg.n_adaptive) return SDSAT_EINVAL;
+  if (draft_table_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
+  return launch_build_block(mode, prev_out_dev, prev_acc_dev, draft_table_dev, table_stride, kv->len, c->adaptive,
+                            b, q, tokens_out_dev, c->stream, true) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_get_error(sdsat_ctx* c, uint32_t* flags) {
+  if (!c) return SDSAT_EINVAL;
+  uint32_t f = 0;
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return SDSAT_ECUDA;
+  if (cudaMemcpy(&f, c->err, sizeof(f), cudaMemcpyDeviceToHost) != cudaSuccess) return SDSAT_ECUDA;
+  if (cudaMemset(c->err, 0, sizeof(f)) != cudaSuccess) return SDSAT_ECUDA;
+  if (flags) *flags = f;
+  return f ? SDSAT_EDEVICE : SDSAT_OK;
+}
+
+sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev) {
+  if (!c || !x_dev || !y_dev || !aligned16(w_dev) || !aligned16(x_dev)) return SDSAT_EINVAL;
+  if (M < 1 || M > SDSAT_MAX_ROWS || K < 8 || K % 8 || N < 1 || (N + 127) / 128 > MAX_GEMM_TILES)
+    return SDSAT_EINVAL;
+  GemmParams g = gemm_base(c, M);
+  CUtensorMap m;
+  if (!make_wmap(&m, w_dev, N, K)) return SDSAT_ECUDA;
+  set_plain(g, m, N, K);
+  g.x = x_dev;
+  g.x_ld = K;
+  g.epi = EPI_STORE;
+  g.out = y_dev;
+  g.out_ld = N;
+  return launch_gemm(g, c->num_sms, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_dev, const void* v_dev,
+                                const int32_t* len_dev, int b, int q, int H, int hd, int cap, float* out_dev) {
+  if (!c || !q_dev || !k_dev || !v_dev || !len_dev || !out_dev) return SDSAT_EINVAL;
+  if (b < 1 || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS || (hd != 64 && hd != 128) || H < 1 || cap < 1)
+    return SDSAT_EINVAL;
+  // the split-KV workspace was sized at create for SDSAT_MAX_ROWS rows of the model's heads
+  const size_t nch = (size_t)(cap + ATT_CHUNK - 1) / ATT_CHUNK;
+  const size_t have = (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * c->att_nch;
+  if ((size_t)b * q * H * nch * hd > have * c->cfg.head_dim || (size_t)b * q * H * nch > have ||
+      (size_t)b * H > (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads)
+    return SDSAT_EINVAL;
+  AttnParams a;
+  std::memset(&a, 0, sizeof(a));
+  a.Q = q_dev;
+  a.q_ld = H * hd;
+  a.k = static_cast<const __nv_bfloat16*>(k_dev);
+  a.v = static_cast<const __nv_bfloat16*>(v_dev);
+  a.len = len_dev;
+  a.seq0 = 0;
+  a.nb = b;
+  a.q = q;
+  a.H = H;
+  a.hd = hd;
+  a.cap = cap;
+  a.out = out_dev;
+  a.out_ld = H * hd;
+  a.part_o = c->att_part_o;
+  a.part_ml = c->att_part_ml;
+  a.nch_max = (cap + ATT_CHUNK - 1) / ATT_CHUNK;
+  a.counters = c->att_counters;
+  a.err = c->err;
+  return launch_attention(a, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_op_exp(sdsat_ctx* c, const float* in_dev, float* out_dev, int n) {
+  if (!c || !in_dev || !out_dev || n < 0) return SDSAT_EINVAL;
+  if (n == 0) return SDSAT_OK;
+  return launch_exp(in_dev, out_dev, n, c->stream) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+}
+
+}  // extern "C"

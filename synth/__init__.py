@@ -167,6 +167,18 @@ def normal_bf16(seed: int, stream: int, shape: Sequence[int], std: float,
     return out
 
 
+def normal_f32(seed: int, stream: int, shape: Sequence[int], std: float = 1.0, device="cpu") -> torch.Tensor:
+    """fp32 tensor ~ N(0, std) (same Irwin-Hall construction, not rounded to bf16)."""
+    shape = tuple(int(s) for s in shape)
+    n = int(math.prod(shape))
+    idx = torch.arange(n, dtype=torch.int64, device=device)
+    a = u32(seed, stream, 2 * idx)
+    b = u32(seed, stream, 2 * idx + 1)
+    s = (a & 0xFFFF) + (a >> 16) + (b & 0xFFFF) + (b >> 16) - 131070
+    scale = torch.tensor(std * math.sqrt(3.0) / 65536.0, dtype=torch.float32, device=device)
+    return (s.to(torch.float32) * scale).reshape(shape)
+
+
 def ones_bf16(n: int, device="cpu") -> torch.Tensor:
     return torch.ones(n, dtype=torch.bfloat16, device=device)
 

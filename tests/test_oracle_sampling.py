@@ -61,10 +61,10 @@ def test_argmax_ties_and_nan():
     assert S.argmax_lowest(np.float32([-np.inf, -np.inf]))[0] == 0
 
 
-def test_int_weights_top_is_2_40():
+def test_int_weights_top_is_2_24():
     l = np.random.default_rng(1).normal(0, 1.3, 500).astype(np.float32)
     W, _ = S.int_weights(l, 0.7)
-    assert int(W.max()) == 1 << 40 and int(np.argmax(W)) == int(np.argmax(l))
+    assert int(W.max()) == 1 << 24 and int(np.argmax(W)) == int(np.argmax(l))
 
 
 def _brute_min_cardinality(W, p_fixed):
@@ -151,6 +151,18 @@ def test_low_temperature_is_greedy():
         g, _ = S.argmax_lowest(l)
         s, _ = S.nucleus_sample(l, 1e-4, 0.95, seed=i, position=i, seq=0)
         assert s == g
+
+
+def test_weights_are_floor_of_scaled_exp():
+    """W_i = floor(e^{(l_i - max)/T} * 2^24) to within the exp's few-ulp error: compare with
+    the exact double-precision value (the floor can move by at most 1)."""
+    rng = np.random.default_rng(5)
+    l = rng.normal(0, 2.0, 4000).astype(np.float32)
+    for T in (0.2, 1.0):
+        W, _ = S.int_weights(l, T)
+        s = ((l - l.max()) / np.float32(T)).astype(np.float32).astype(np.float64)
+        exact = np.floor(np.exp(s) * 2.0**24)
+        assert np.abs(W.astype(np.float64) - exact).max() <= 1.0
 
 
 def test_degenerate_rows():
