@@ -1,0 +1,581 @@
+#!/usr/bin/env python3
+"""Benchmark: SDSAT two-step-draft-then-verify decoding on GB300 (one JSON line).
+
+A step is one block decode step: build the block input, one block forward of
+q = k + 1 positions through every layer, target selection + Eq. 3 verification
++ KV commit.  Steps alternate draft step 1 / draft step 2 (Sec. 2.1.1); a
+generation is the steps that emit `new` tokens per sequence after a `prompt`
+of uniform ids, and generations run back to back.  Drafts come from a seeded
+per-position stub that copies the model's own plain-decoding token with the
+workload's match rate (random weights cannot draft).
+
+value      generated tokens/s, the loop replayed from CUDA graphs, inputs and
+           state resident in HBM (weights 13-26 GB > L2, so no flush needed).
+e2e        the same metric through the C ABI with host buffers: each step the
+           host builds the block input, copies it in (pinned -> device), runs the
+           step, copies the emitted tokens back and reads them.
+roofline   the skinny GEMM (the dominant kernel): algorithmic bytes / CUDA-event
+           time of its launches in a profiled pass, against the measured HBM
+           copy bandwidth.
+cpu_baseline / --impl reference   the CPU oracle timed on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "generated tokens/s at bs1 (7B/13B shape); verify-step HBM GB/s vs 8 TB/s"
+NOMINAL_HBM_GBS = 8000.0
+
+WORKLOADS = {
+    # CodeLlama-7B shape, greedy, prompt 2048, 256 new tokens, k = 5, stub match 0.7
+    "7b": dict(shape="7b", batch=1, prompt=2048, new=256, k=5, temperature=0.0, top_p=1.0, top_k=0, match=0.7),
+    # CodeLlama-13B shape, greedy, prompt 4096
+    "13b": dict(shape="13b", batch=1, prompt=4096, new=256, k=5, temperature=0.0, top_p=1.0, top_k=0, match=0.7),
+    # 7B shape, nucleus verification (top_p 0.95, T 0.2), batch 4, prompts of 1024
+    "7b-nucleus": dict(shape="7b", batch=4, prompt=1024, new=256, k=5, temperature=0.2, top_p=0.95, top_k=0,
+                       match=0.6),
+    # tiny correctness shape
+    "tiny": dict(shape="tiny", batch=1, prompt=128, new=64, k=5, temperature=0.0, top_p=1.0, top_k=0, match=0.7),
+}
+
+
+def expected_tokens_per_step(k: int, match: float) -> float:
+    """Two steps emit 2 + m tokens, m = leading matches of k drafts (Sec. 2.1.1)."""
+    return (2.0 + sum(match ** j for j in range(1, k + 1))) / 2.0
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.proc = None
+        self.uuid = uuid
+
+    def start(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-lms", "100"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            return None
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- bytes
+def gemm_bytes(shape, M):
+    """Algorithmic HBM bytes of one launch of each projection (weights + activations + outputs)."""
+    d, F, R, V = shape.d_model, shape.ffn_dim, shape.n_heads * shape.head_dim, shape.vocab
+    return {
+        "gemm_qkv": 3 * R * d * 2 + M * d * 4 + M * R * 4 + 2 * M * R * 2,
+        "gemm_o": d * R * 2 + M * R * 4 + 2 * M * d * 4,
+        "gemm_gateup": 2 * F * d * 2 + M * d * 4 + M * F * 4,
+        "gemm_down": d * F * 2 + M * F * 4 + 2 * M * d * 4,
+        "gemm_lm_head": V * d * 2 + M * d * 4 + M * V * 4,
+    }
+
+
+def weight_bytes(shape):
+    d, F, R, V, L = shape.d_model, shape.ffn_dim, shape.n_heads * shape.head_dim, shape.vocab, shape.n_layers
+    return L * (4 * R * d + 3 * F * d) * 2 + 2 * V * d * 2
+
+
+def kv_bytes_per_layer_slot(shape):
+    return 2 * shape.n_heads * shape.head_dim * 2
+
+
+# ----------------------------------------------------------------------------- our arm
+class Runner:
+    def __init__(self, wl, device):
+        import torch
+        import synth
+        import paper_2403_18647_gb300 as sd
+        self.torch, self.synth, self.sd = torch, synth, sd
+        self.wl = wl
+        self.shape = synth.SHAPES[wl["shape"]]
+        self.b, self.k = wl["batch"], wl["k"]
+        self.q = self.k + 1
+        self.P = wl["prompt"]
+        self.new = wl["new"]
+        self.cap = self.P + 2 * self.new + 8 * self.q
+        self.dev = device
+        self.weights = synth.make_model(self.shape, seed=0, device=device)
+        torch.cuda.synchronize()
+        self.ctx = sd.Context(self.shape, self.weights, max_position=self.cap + 64)
+        self.kv = self.ctx.kv(self.b, self.cap)
+        V = self.shape.vocab
+        self.logits = torch.empty(self.b * self.q, V, device=device)
+        self.toks = torch.zeros(self.b * self.q, dtype=torch.int32, device=device)
+        self.acc = torch.ones(self.b, dtype=torch.int32, device=device)
+        self.out = torch.zeros(self.b * self.q, dtype=torch.int32, device=device)
+        self.prompts = [synth.prompt_ids(0, s, self.P, self.shape.adaptive_id, device) for s in range(self.b)]
+        for s in range(self.b):
+            self.ctx.prefill(self.kv, s, self.prompts[s][:-1].contiguous())
+        self.init_out = torch.zeros_like(self.out)
+        for s in range(self.b):
+            self.init_out[s * self.q] = self.prompts[s][-1]
+        self.init_acc = torch.ones_like(self.acc)
+        self.start_len = torch.full((self.b,), self.P - 1, dtype=torch.int32, device=device)
+        self._make_table()
+        torch.cuda.synchronize()
+
+    # target selection for this workload
+    def accept(self, n_verify, commit=True):
+        wl = self.wl
+        if wl["temperature"] > 0:
+            self.ctx.accept_nucleus(self.kv, self.logits, self.toks, self.b, self.q, n_verify, wl["top_p"],
+                                    wl["temperature"], 1234, self.acc, self.out, top_k=wl["top_k"], commit=commit)
+        else:
+            self.ctx.accept_greedy(self.kv, self.logits, self.toks, self.b, self.q, n_verify, self.acc, self.out,
+                                   commit=commit)
+
+    def _make_table(self):
+        """Plain decoding (q = 1) from the prompt gives each position's reference token; the stub
+        table holds it with the workload's match rate, else a uniform id."""
+        torch = self.torch
+        n_ref = 2 * self.new + 8 * self.q
+        ref = torch.zeros(n_ref, self.b, dtype=torch.int32, device=self.dev)
+        lg = torch.empty(self.b, self.shape.vocab, device=self.dev)
+        tok = self.init_out.view(self.b, self.q)[:, 0].contiguous()
+        acc = torch.empty(self.b, dtype=torch.int32, device=self.dev)
+        wl = self.wl
+        n_run = min(n_ref, self.cap - self.P)
+        for i in range(n_run):
+            self.ctx.block_forward(self.kv, tok, lg, self.b, 1)
+            if wl["temperature"] > 0:
+                self.ctx.accept_nucleus(self.kv, lg, tok, self.b, 1, 0, wl["top_p"], wl["temperature"], 1234, acc,
+                                        tok, top_k=wl["top_k"])
+            else:
+                self.ctx.accept_greedy(self.kv, lg, tok, self.b, 1, 0, acc, tok)
+            ref[i] = tok
+        self.ctx.kv_commit(self.kv, self.start_len, self.b)
+        self.stride = self.cap + 32
+        table = torch.zeros(self.b, self.stride, dtype=torch.int32, device=self.dev)
+        for s in range(self.b):
+            full = torch.zeros(self.stride, dtype=torch.int32, device=self.dev)
+            full[self.P:self.P + n_run] = ref[:n_run, s]
+            table[s] = self.synth.stub_table(0, s, full, wl["match"], self.shape.vocab)
+        self.table = table.contiguous()
+        self.ref = ref
+
+    def reset(self):
+        self.ctx.kv_commit(self.kv, self.start_len, self.b)
+        self.out.copy_(self.init_out)
+        self.acc.copy_(self.init_acc)
+
+    def step(self, mode):
+        self.ctx.build_block(self.kv, mode, self.out, self.acc, self.toks, self.b, self.q,
+                             draft_table=self.table if mode == 2 else None, table_stride=self.stride)
+        self.ctx.block_forward(self.kv, self.toks, self.logits, self.b, self.q)
+        self.accept(0 if mode == 1 else self.k)
+
+    def calibrate(self):
+        """One generation with host checks: the number of steps it takes and the tokens
+        and committed lengths of every step (for the byte counts)."""
+        torch = self.torch
+        self.reset()
+        base = self.ctx.kv_emitted(self.kv).clone()
+        lens, toks = [], []
+        n = 0
+        while True:
+            lens.append(self.ctx.kv_lengths(self.kv).cpu().tolist())
+            self.step(1 if n % 2 == 0 else 2)
+            n += 1
+            em = (self.ctx.kv_emitted(self.kv) - base).cpu().tolist()
+            toks.append(sum(em) - sum(toks))
+            if n % 2 == 0 and min(em) >= self.new:
+                break
+        flags = self.ctx.get_error()
+        return n, lens, toks, flags
+
+    def capture(self):
+        torch = self.torch
+        try:
+            graphs = []
+            s = torch.cuda.Stream()
+            s.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(s):
+                for mode in (1, 2):           # warm the path on the capture stream
+                    self.step(mode)
+            torch.cuda.current_stream().wait_stream(s)
+            torch.cuda.synchronize()
+            for mode in (1, 2):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    self.step(mode)
+                graphs.append(g)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                self.reset()
+            graphs.append(g)
+            torch.cuda.synchronize()
+            return graphs
+        except Exception as e:  # graphs are an optimisation; eager launches run the same kernels
+            print("note: CUDA graph capture failed (%s); timing eager launches" % e, file=sys.stderr)
+            torch.cuda.synchronize()
+            return None
+
+    def run_steps(self, n, steps_per_gen, graphs, start=0):
+        """n steps of back-to-back generations, starting at global step index `start`."""
+        for i in range(start, start + n):
+            j = i % steps_per_gen
+            if j == 0 and i > 0:
+                graphs[2].replay() if graphs else self.reset()
+            if graphs:
+                graphs[j % 2].replay()
+            else:
+                self.step(1 if j % 2 == 0 else 2)
+
+
+def run_ours(args, wl, rank, world):
+    import torch
+    import torch.distributed as dist
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    r = Runner(wl, dev)
+    shape = r.shape
+    steps_per_gen, lens, toks_cal, flags = r.calibrate()
+    # schedule the timed region as whole-generation-aligned steps
+    graphs = r.capture()
+    r.reset()
+    r.run_steps(args.warmup, steps_per_gen, graphs)
+    r.reset()
+    torch.cuda.synchronize()
+    em0 = r.ctx.kv_emitted(r.kv).sum().item()
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    clocks = ClockSampler(uuid)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    r.run_steps(args.steps, steps_per_gen, graphs)
+    e1.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    tokens = r.ctx.kv_emitted(r.kv).sum().item() - em0
+    flags |= r.ctx.get_error()
+    if world > 1:
+        t = torch.tensor([ms, float(tokens)], device=dev)
+        mx = t.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        ms, tokens = mx[0].item(), t[1].item()
+    value = tokens / (ms / 1e3)
+    # --- profiled pass (per-kernel CUDA events; launches serialised) for the roofline
+    r.reset()
+    n_prof = min(args.steps, steps_per_gen)
+    launches_per_step = 4 + 5 * shape.n_layers
+    r.ctx.profile_begin(n_prof * (launches_per_step + 2) + 16)
+    r.run_steps(n_prof, steps_per_gen, None)
+    kstats = r.ctx.profile_end()
+    # --- e2e: the C ABI with host buffers (host builds inputs, reads outputs every step)
+    e2e = run_e2e(r, args.steps, steps_per_gen)
+    # --- bytes
+    M = r.b * r.q
+    gb = gemm_bytes(shape, M)
+    g_bytes = sum(gb[n] * kstats.get(n, (0, 0))[0] for n in gb)
+    g_ms = sum(kstats.get(n, (0, 0.0))[1] for n in gb)
+    g_launches = sum(kstats.get(n, (0, 0))[0] for n in gb)
+    peak, peak_kind = peaks()
+    achieved = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else 0.0
+    # per-step algorithmic bytes over one calibrated generation
+    Wb = weight_bytes(shape)
+    slot = kv_bytes_per_layer_slot(shape) * shape.n_layers
+    kv_read = [sum(l + r.q for l in ln) * slot for ln in lens]
+    kv_write = M * slot
+    logit_b = M * shape.vocab * 4
+    step_bytes = Wb + statistics.mean(kv_read) + kv_write + logit_b
+    ms_step = ms / args.steps
+    step_gbs = step_bytes / (ms_step / 1e3) / 1e9
+    # --- gpu launches in the timed region: our kernels only
+    resets = sum(1 for i in range(args.steps) if i % steps_per_gen == 0 and i > 0)
+    gpu_launches = args.steps * launches_per_step + resets
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed 0)",
+                   "global_batch": r.b * world, "seq_len": r.P, "new_tokens": r.new, "k": r.k, "q": r.q,
+                   "draft_stub_match": wl["match"], "temperature": wl["temperature"], "top_p": wl["top_p"],
+                   "parallelism": "replicas%d" % world if world > 1 else "single",
+                   "l2": "inputs larger than L2 (%.1f GB of weights streamed per step)" % (Wb / 1e9),
+                   "graphs": graphs is not None, "mma": "bf16 hi+lo activations x bf16 weights -> fp32"},
+        "tokens_per_step": round(tokens / world / args.steps, 4),
+        "expected_tokens_per_step": round(expected_tokens_per_step(r.k, wl["match"]), 4),
+        "steps_per_generation": steps_per_gen,
+        "step_hbm": {"bytes": int(step_bytes), "achieved_gbs": round(step_gbs, 1),
+                     "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4),
+                     "frac_of_measured": round(step_gbs / peak, 4)},
+        "roofline": {"kernel": "skinny_gemm (all projections)", "bound": "hbm", "achieved": round(achieved, 1),
+                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak_source": peak_kind, "launches": g_launches,
+                     "bytes_per_launch": int(g_bytes / max(1, g_launches)),
+                     "ms_per_launch": round(g_ms / max(1, g_launches), 5)},
+        "kernels": {k: {"launches": v[0], "ms_total": round(v[1], 4), "us_per_launch": round(1e3 * v[1] / v[0], 2)}
+                    for k, v in kstats.items()},
+        "e2e": e2e, "gpu_launches": gpu_launches, "device_error_flags": flags,
+    }
+    if clk:
+        out["clocks"] = clk
+    return r, out
+
+
+def run_e2e(r, steps, steps_per_gen):
+    """The decode loop a host program writes against the C ABI: every step the host builds
+    the block input from the previous step's emitted tokens (pinned buffer -> device copy),
+    calls block_forward and accept, copies the emitted tokens and accepted lengths back and
+    reads them before the next step."""
+    import torch
+    b, q, k = r.b, r.q, r.k
+    tok_h = torch.zeros(b * q, dtype=torch.int32).pin_memory()
+    out_h = torch.zeros(b * q, dtype=torch.int32).pin_memory()
+    acc_h = torch.zeros(b, dtype=torch.int32).pin_memory()
+    table = r.table.cpu()
+    adaptive = [r.shape.adaptive_id] * k
+    r.reset()
+    torch.cuda.synchronize()
+    lens = [r.P - 1] * b
+    last_out = [[int(r.prompts[s][-1])] + [0] * k for s in range(b)]
+    last_acc = [1] * b
+    tokens = 0
+    st = torch.cuda.current_stream()
+    t0 = time.perf_counter()
+    for i in range(steps):
+        j = i % steps_per_gen
+        if j == 0 and i > 0:
+            r.reset()
+            lens = [r.P - 1] * b
+            last_out = [[int(r.prompts[s][-1])] + [0] * k for s in range(b)]
+            last_acc = [1] * b
+        mode = 1 if j % 2 == 0 else 2
+        blk = []
+        for s in range(b):
+            if mode == 1:
+                blk += [last_out[s][last_acc[s] - 1]] + adaptive
+            else:
+                blk += [last_out[s][0]] + [int(table[s, lens[s] + jj]) for jj in range(1, q)]
+        tok_h.copy_(torch.tensor(blk, dtype=torch.int32))
+        r.toks.copy_(tok_h, non_blocking=True)
+        r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
+        r.accept(0 if mode == 1 else k)
+        out_h.copy_(r.out, non_blocking=True)
+        acc_h.copy_(r.acc, non_blocking=True)
+        st.synchronize()
+        o = out_h.tolist()
+        a = acc_h.tolist()
+        for s in range(b):
+            last_out[s] = o[s * q:(s + 1) * q]
+            last_acc[s] = a[s]
+            lens[s] += a[s]
+        tokens += sum(a)
+    t1 = time.perf_counter()
+    return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": b * q * 4,
+            "d2h_bytes_per_step": b * q * 4 + b * 4, "launch": "eager C-ABI calls, host sync each step"}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def oracle_sample(shape_name, wl, weights_gpu=None, n_layers=2, repeat=1, gen_device="cpu"):
+    """Time the CPU oracle on a bounded sample of one block step at the workload's shape:
+    `n_layers` decoder layers (their weights widened once and cached, as the oracle does)
+    against a synthetic KV of the prompt length, plus the final norm + LM head, then
+    extrapolate to all layers.  Returns (seconds per full step, details)."""
+    import numpy as np
+    import torch
+    import synth
+    from oracle import model as OM
+    shape = synth.SHAPES[shape_name]
+    q = wl["k"] + 1
+    P = wl["prompt"]
+
+    def provider(name, layer):
+        if weights_gpu is not None:
+            t = weights_gpu[name] if layer < 0 else weights_gpu["layers"][layer][name]
+            return t.cpu()
+        return synth.make_weight(shape, name, layer, 0, "cpu")
+
+    W = OM.Weights(shape, provider=provider, cache=True)
+    small = synth.ModelShape("sample", n_layers, shape.d_model, shape.n_heads, shape.head_dim, shape.ffn_dim,
+                             shape.vocab, shape.adaptive_id)
+    kv = OM.KVCache(small, 1, P + q)
+    for l in range(n_layers):
+        for which, dst in ((0, kv.K), (1, kv.V)):
+            vals = synth.kv_values(0, l, which, (shape.n_heads, P, shape.head_dim), device=gen_device)
+            dst[l][0][:, :P] = vals.cpu().double().numpy()
+    kv.len[0] = P
+    toks = synth.uniform_ids(0, 999, q, shape.adaptive_id).tolist()
+    # widen the sampled weights once (the oracle caches them)
+    for l in range(n_layers):
+        for n in synth.LAYER_MATS:
+            W.get(n, l)
+    for n in ("embed", "final_norm", "lm_head"):
+        W.get(n)
+    t0 = time.perf_counter()
+    for _ in range(repeat):
+        OM.block_forward(W, kv, 0, toks, layers=range(n_layers), final=False)
+    t_layers = (time.perf_counter() - t0) / repeat
+    t0 = time.perf_counter()
+    OM.block_forward(W, kv, 0, toks, layers=[], final=True)
+    t_head = time.perf_counter() - t0
+    per_layer = t_layers / n_layers
+    return shape.n_layers * per_layer + t_head, {"per_layer_s": per_layer, "head_s": t_head}
+
+
+def cpu_baseline(args, wl, weights_gpu):
+    tps = expected_tokens_per_step(wl["k"], wl["match"])
+    dev = next(iter(weights_gpu["layers"][0].values())).device if weights_gpu is not None else "cpu"
+    t_step, det = oracle_sample(wl["shape"], wl, weights_gpu, n_layers=2, gen_device=dev)
+    return {"value": round(tps / t_step, 4), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": ("one q=%d block step at context %d: 2 of %d decoder layers timed (weights widened and cached "
+                       "first) plus the final norm + LM head, extrapolated to all layers (%.2f s/layer, %.2f s head); "
+                       "tokens/step = %.3f, the stub's expectation" %
+                       (wl["k"] + 1, wl["prompt"], __import__("synth").SHAPES[wl["shape"]].n_layers,
+                        det["per_layer_s"], det["head_s"], tps)),
+            "s_per_step": round(t_step, 3)}
+
+
+def run_reference(args, wl, rank, world):
+    """The reference arm: the CPU oracle (no reference implementation exists).  Each step is a
+    bounded sample -- one decoder layer of the block step -- scaled by the layer count."""
+    import synth
+    from oracle import model as OM
+    shape = synth.SHAPES[wl["shape"]]
+    tps = expected_tokens_per_step(wl["k"], wl["match"])
+    q = wl["k"] + 1
+    P = wl["prompt"]
+    W = OM.Weights(shape, provider=lambda n, l: synth.make_weight(shape, n, l, 0, "cpu"), cache=True)
+    small = synth.ModelShape("sample", 1, shape.d_model, shape.n_heads, shape.head_dim, shape.ffn_dim,
+                             shape.vocab, shape.adaptive_id)
+    kv = OM.KVCache(small, 1, P + q)
+    kv.K[0][0][:, :P] = synth.kv_values(0, 0, 0, (shape.n_heads, P, shape.head_dim)).double().numpy()
+    kv.V[0][0][:, :P] = synth.kv_values(0, 0, 1, (shape.n_heads, P, shape.head_dim)).double().numpy()
+    kv.len[0] = P
+    toks = synth.uniform_ids(0, 999, q, shape.adaptive_id).tolist()
+    for n in synth.LAYER_MATS:
+        W.get(n, 0)
+    for n in ("embed", "final_norm", "lm_head"):
+        W.get(n)
+    t0 = time.perf_counter()
+    OM.block_forward(W, kv, 0, toks, layers=[], final=True)
+    t_head = time.perf_counter() - t0
+    for _ in range(args.warmup):
+        OM.block_forward(W, kv, 0, toks, layers=[0], final=False)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        OM.block_forward(W, kv, 0, toks, layers=[0], final=False)
+        times.append(time.perf_counter() - t0)
+    per_layer = statistics.mean(times)
+    t_step = shape.n_layers * per_layer + t_head
+    value = tps / t_step
+    sample = ("each step: one decoder layer of a q=%d block step at context %d (weights widened once and cached), "
+              "scaled by %d layers, plus the final norm + LM head timed once (%.2f s); tokens/step = %.3f, the "
+              "stub's expectation" % (q, P, shape.n_layers, t_head, tps))
+    return {"metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(t_step * 1e3, 2), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed 0)",
+                       "global_batch": wl["batch"], "seq_len": P, "k": wl["k"]},
+            "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="7b", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    wl = WORKLOADS[args.config]
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, wl, rank, world)), flush=True)
+        return
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0"))))
+    r, out = run_ours(args, wl, rank, world)
+    if rank == 0:
+        if not args.no_cpu_baseline:
+            try:
+                out["cpu_baseline"] = cpu_baseline(args, wl, r.weights)
+            except Exception as e:  # keep the GPU line even if the host runs out of memory
+                out["cpu_baseline"] = {"value": None, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                                       "sample": "failed: %s" % e}
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -205,6 +205,12 @@ SDSAT_API sdsat_status sdsat_kv_commit(sdsat_ctx* ctx, sdsat_kv* kv, const int32
  * asynchronously.  Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_kv_lengths(sdsat_ctx* ctx, const sdsat_kv* kv, int32_t* lens_dev, int b);
 
+/* Tokens emitted so far per sequence: every accept call with commit != 0 adds
+ * 1 + m to emitted[s] on the device.  Copies emitted[0 .. b-1] into
+ * emitted_dev (int64 [b]) and, when reset != 0, zeroes the counters after the
+ * copy.  Asynchronous.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_kv_emitted(sdsat_ctx* ctx, sdsat_kv* kv, int64_t* emitted_dev, int b, int reset);
+
 /* Build the next block input on the device (the block inputs of Eq. 1 and Eq. 2),
  * so that a whole loop runs without the host:
  *   mode 1 (draft step 1): row 0 = prev_out[s*q + prev_acc[s] - 1] (the newest
@@ -250,6 +256,24 @@ SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, co
 
 /* out[i] = the nucleus sampler's exp (see sdsat_accept_nucleus) of in[i] <= 0. */
 SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* out_dev, int n);
+
+/* ---- measurement ------------------------------------------------------------------ */
+
+/* Per-kernel timing: between sdsat_profile_begin and sdsat_profile_end every
+ * kernel the library launches on ctx is bracketed by CUDA events recorded on
+ * the context stream (which serialises the launches: no overlap between
+ * consecutive kernels while profiling).  begin creates a pool of events for
+ * up to max_launches launches (call it outside any graph capture); launches
+ * past the pool are not timed.  end synchronises and returns one record per
+ * kernel class that ran: its name, launch count and summed duration. */
+typedef struct {
+  char name[32];
+  int64_t launches;
+  double total_ms;
+} sdsat_kernel_stat;
+
+SDSAT_API sdsat_status sdsat_profile_begin(sdsat_ctx* ctx, int max_launches);
+SDSAT_API sdsat_status sdsat_profile_end(sdsat_ctx* ctx, sdsat_kernel_stat* out, int max_out, int* n_out);
 
 #ifdef __cplusplus
 }

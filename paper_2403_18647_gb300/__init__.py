@@ -44,6 +44,10 @@ class Config(ctypes.Structure):
                 ("adaptive_ids", ctypes.c_int32 * MAX_ADAPTIVE)]
 
 
+class KernelStat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int64), ("total_ms", ctypes.c_double)]
+
+
 class LayerWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down")]
@@ -77,6 +81,9 @@ def _lib():
             "sdsat_accept_nucleus": [P, P, P, P, I, I, I, F, F, U64, I, P, P, I],
             "sdsat_kv_commit": [P, P, P, I],
             "sdsat_kv_lengths": [P, P, P, I],
+            "sdsat_kv_emitted": [P, P, P, I, I],
+            "sdsat_profile_begin": [P, I],
+            "sdsat_profile_end": [P, ctypes.POINTER(KernelStat), I, ctypes.POINTER(I)],
             "sdsat_build_block": [P, P, I, P, P, P, I, I, I, P],
             "sdsat_prefill": [P, P, I, P, I],
             "sdsat_get_error": [P, ctypes.POINTER(ctypes.c_uint32)],
@@ -244,6 +251,25 @@ class Context:
         self._bind_stream()
         _check(_lib().sdsat_kv_lengths(self.handle, kv.handle, _ptr(out), b), "sdsat_kv_lengths")
         return out
+
+    def kv_emitted(self, kv: KV, reset: bool = False):
+        """Tokens emitted per sequence so far (int64 CUDA tensor [batch])."""
+        import torch
+        out = torch.empty(kv.batch, dtype=torch.int64, device="cuda")
+        self._bind_stream()
+        _check(_lib().sdsat_kv_emitted(self.handle, kv.handle, _ptr(out), kv.batch, int(reset)), "sdsat_kv_emitted")
+        return out
+
+    def profile_begin(self, max_launches: int):
+        _check(_lib().sdsat_profile_begin(self.handle, max_launches), "sdsat_profile_begin")
+
+    def profile_end(self) -> dict:
+        """{kernel class: (launches, total_ms)} of the launches since profile_begin."""
+        self._bind_stream()
+        buf = (KernelStat * 32)()
+        n = ctypes.c_int(0)
+        _check(_lib().sdsat_profile_end(self.handle, buf, 32, ctypes.byref(n)), "sdsat_profile_end")
+        return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].total_ms)) for i in range(n.value)}
 
     def build_block(self, kv: KV, mode: int, prev_out, prev_acc, tokens_out, b: int, q: int,
                     draft_table=None, table_stride: int = 0):

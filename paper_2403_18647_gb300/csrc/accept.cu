@@ -373,6 +373,7 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
     const int nl = __ldcg(p.len + s) + 1 + m;
     if (nl <= p.cap) p.len[s] = nl;
     else set_error(p.err, ERR_CAPACITY);
+    if (p.emitted) p.emitted[s] += 1 + m;
   }
   p.counters[sl] = 0;
 }

@@ -101,6 +101,7 @@ struct AcceptParams {
   int* out_tokens;          // [nb*q]
   int* targets;             // scratch [nb*q]
   int* counters;            // scratch [nb], zero between launches
+  long long* emitted;       // [B] tokens emitted per sequence (commit only), or null
   uint32_t* err;
 };
 cudaError_t launch_accept(const AcceptParams& p, cudaStream_t st, bool pdl);

@@ -55,6 +55,15 @@ struct LayerMaps {
   CUtensorMap q, k, v, o, gate, up, down;
 };
 
+// kernel classes for the profiling hook
+enum KClass : int {
+  K_EMBED = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
+  K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_COUNT
+};
+const char* const KCLASS_NAME[K_COUNT] = {"embed", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
+                                          "gemm_lm_head", "accept", "build_block", "kv_commit", "prefill_commit",
+                                          "gemm_op", "attention_op"};
+
 constexpr int MAX_GEMM_TILES = 1 << 16;
 
 }  // namespace
@@ -85,6 +94,11 @@ struct sdsat_ctx {
   int* adaptive = nullptr;
   uint32_t* err = nullptr;
   std::vector<void*> allocs;
+  // profiling hook
+  bool prof = false;
+  std::vector<cudaEvent_t> prof_events;
+  std::vector<int> prof_class;
+  size_t prof_used = 0;
 };
 
 struct sdsat_kv {
@@ -93,9 +107,22 @@ struct sdsat_kv {
   __nv_bfloat16* k = nullptr;
   __nv_bfloat16* v = nullptr;
   int* len = nullptr;
+  long long* emitted = nullptr;
 };
 
 namespace {
+
+// Run one kernel launch, bracketed by profiling events when the hook is on.
+template <typename F>
+cudaError_t timed(sdsat_ctx* c, int cls, F&& launch) {
+  if (!c->prof || 2 * (c->prof_used + 1) > c->prof_events.size()) return launch();
+  const size_t i = c->prof_used++;
+  cudaEventRecord(c->prof_events[2 * i], c->stream);
+  const cudaError_t e = launch();
+  cudaEventRecord(c->prof_events[2 * i + 1], c->stream);
+  c->prof_class[i] = cls;
+  return e;
+}
 
 template <typename T>
 bool dalloc(sdsat_ctx* c, T** p, size_t count) {
@@ -151,8 +178,10 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
   const int M = nb * q, d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd;
   cudaStream_t st = c->stream;
   const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
-  if (launch_embed(tokens, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, d, M, c->h, c->err, st,
-                   true) != cudaSuccess)
+  if (timed(c, K_EMBED, [&] {
+        return launch_embed(tokens, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, d, M, c->h, c->err,
+                            st, true);
+      }) != cudaSuccess)
     return SDSAT_ECUDA;
   for (int l = 0; l < cf.n_layers; ++l) {
     const sdsat_layer_weights& W = c->layers[l];
@@ -186,7 +215,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.positions = positions;
     g.rope = c->rope;
     g.rope_len = cf.max_position;
-    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
     // block-causal attention
     AttnParams a;
     std::memset(&a, 0, sizeof(a));
@@ -208,7 +237,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
     a.counters = c->att_counters;
     a.err = c->err;
-    if (launch_attention(a, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
     // O projection + residual
     g = gemm_base(c, M);
     set_plain(g, mp.o, d, R);
@@ -217,7 +246,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
-    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
     // gate/up with the fused RMSNorm and SiLU(gate) * up
     g = gemm_base(c, M);
     g.tmap[0] = mp.gate;
@@ -234,7 +263,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_SWIGLU;
     g.out = c->act;
     g.out_ld = F;
-    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
     // down projection + residual
     g = gemm_base(c, M);
     set_plain(g, mp.down, d, F);
@@ -243,7 +272,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
-    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
   }
   if (logits) {
     GemmParams g = gemm_base(c, M);
@@ -255,7 +284,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_STORE;
     g.out = logits;
     g.out_ld = cf.vocab;
-    if (launch_gemm(g, c->num_sms, st, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
   }
   return SDSAT_OK;
 }
@@ -291,7 +320,9 @@ sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, cons
   p.targets = c->acc_targets;
   p.counters = c->acc_counters;
   p.err = c->err;
-  return launch_accept(p, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+  p.emitted = kv->emitted;
+  return timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+                                                                                          : SDSAT_ECUDA;
 }
 
 }  // namespace
@@ -314,6 +345,7 @@ const char* sdsat_status_string(sdsat_status s) {
 void sdsat_destroy(sdsat_ctx* c) {
   if (!c) return;
   cudaStreamSynchronize(c->stream);
+  for (cudaEvent_t e : c->prof_events) cudaEventDestroy(e);
   for (void* p : c->allocs) cudaFree(p);
   delete c;
 }
@@ -416,23 +448,27 @@ sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** ou
   kv->batch = batch;
   kv->cap = max_len;
   const size_t n = (size_t)c->cfg.n_layers * batch * c->cfg.n_heads * max_len * c->cfg.head_dim;
-  void *k = nullptr, *v = nullptr, *len = nullptr;
+  void *k = nullptr, *v = nullptr, *len = nullptr, *em = nullptr;
   if (cudaMalloc(&k, n * 2) != cudaSuccess || cudaMalloc(&v, n * 2) != cudaSuccess ||
-      cudaMalloc(&len, batch * sizeof(int)) != cudaSuccess) {
+      cudaMalloc(&len, batch * sizeof(int)) != cudaSuccess || cudaMalloc(&em, batch * sizeof(long long)) != cudaSuccess) {
     cudaFree(k);
     cudaFree(v);
     cudaFree(len);
+    cudaFree(em);
     delete kv;
     return SDSAT_ENOMEM;
   }
   if (cudaMemset(k, 0, n * 2) != cudaSuccess || cudaMemset(v, 0, n * 2) != cudaSuccess ||
-      cudaMemset(len, 0, batch * sizeof(int)) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+      cudaMemset(len, 0, batch * sizeof(int)) != cudaSuccess ||
+      cudaMemset(em, 0, batch * sizeof(long long)) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
     cudaFree(k);
     cudaFree(v);
     cudaFree(len);
+    cudaFree(em);
     delete kv;
     return SDSAT_ECUDA;
   }
+  kv->emitted = static_cast<long long*>(em);
   kv->k = static_cast<__nv_bfloat16*>(k);
   kv->v = static_cast<__nv_bfloat16*>(v);
   kv->len = static_cast<int*>(len);
@@ -446,6 +482,7 @@ void sdsat_kv_destroy(sdsat_kv* kv) {
   cudaFree(kv->k);
   cudaFree(kv->v);
   cudaFree(kv->len);
+  cudaFree(kv->emitted);
   delete kv;
 }
 
@@ -512,7 +549,9 @@ sdsat_status sdsat_prefill(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
     const int qn = std::min(SDSAT_MAX_Q, n - i);
     const sdsat_status s = forward(c, kv, seq, 1, qn, tokens_dev + i, nullptr, nullptr);
     if (s != SDSAT_OK) return s;
-    if (launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, true) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, true); }) !=
+        cudaSuccess)
+      return SDSAT_ECUDA;
   }
   return SDSAT_OK;
 }
@@ -533,8 +572,10 @@ sdsat_status sdsat_accept_nucleus(sdsat_ctx* c, sdsat_kv* kv, const float* logit
 
 sdsat_status sdsat_kv_commit(sdsat_ctx* c, sdsat_kv* kv, const int32_t* new_len_dev, int b) {
   if (!c || !kv || kv->ctx != c || !new_len_dev || b < 1 || b > kv->batch || b > 64) return SDSAT_EINVAL;
-  return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, true) == cudaSuccess ? SDSAT_OK
-                                                                                                 : SDSAT_ECUDA;
+  return timed(c, K_KV_COMMIT, [&] { return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, true); }) ==
+                 cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
 }
 
 sdsat_status sdsat_kv_lengths(sdsat_ctx* c, const sdsat_kv* kv, int32_t* lens_dev, int b) {
@@ -544,6 +585,57 @@ sdsat_status sdsat_kv_lengths(sdsat_ctx* c, const sdsat_kv* kv, int32_t* lens_de
              : SDSAT_ECUDA;
 }
 
+sdsat_status sdsat_kv_emitted(sdsat_ctx* c, sdsat_kv* kv, int64_t* emitted_dev, int b, int reset) {
+  if (!c || !kv || kv->ctx != c || !emitted_dev || b < 1 || b > kv->batch) return SDSAT_EINVAL;
+  if (cudaMemcpyAsync(emitted_dev, kv->emitted, b * sizeof(long long), cudaMemcpyDeviceToDevice, c->stream) !=
+      cudaSuccess)
+    return SDSAT_ECUDA;
+  if (reset && cudaMemsetAsync(kv->emitted, 0, b * sizeof(long long), c->stream) != cudaSuccess) return SDSAT_ECUDA;
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_profile_begin(sdsat_ctx* c, int max_launches) {
+  if (!c || max_launches < 1) return SDSAT_EINVAL;
+  for (cudaEvent_t e : c->prof_events) cudaEventDestroy(e);
+  c->prof_events.assign(2 * (size_t)max_launches, nullptr);
+  for (auto& e : c->prof_events)
+    if (cudaEventCreate(&e) != cudaSuccess) return SDSAT_ECUDA;
+  c->prof_class.assign(max_launches, 0);
+  c->prof_used = 0;
+  c->prof = true;
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_profile_end(sdsat_ctx* c, sdsat_kernel_stat* out, int max_out, int* n_out) {
+  if (!c || !c->prof) return SDSAT_EINVAL;
+  c->prof = false;
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return SDSAT_ECUDA;
+  long long cnt[K_COUNT] = {0};
+  double ms[K_COUNT] = {0};
+  for (size_t i = 0; i < c->prof_used; ++i) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, c->prof_events[2 * i], c->prof_events[2 * i + 1]) != cudaSuccess) return SDSAT_ECUDA;
+    cnt[c->prof_class[i]] += 1;
+    ms[c->prof_class[i]] += t;
+  }
+  int n = 0;
+  for (int k = 0; k < K_COUNT; ++k) {
+    if (!cnt[k]) continue;
+    if (out && n < max_out) {
+      std::memset(&out[n], 0, sizeof(out[n]));
+      std::strncpy(out[n].name, KCLASS_NAME[k], sizeof(out[n].name) - 1);
+      out[n].launches = cnt[k];
+      out[n].total_ms = ms[k];
+    }
+    ++n;
+  }
+  if (n_out) *n_out = n;
+  for (cudaEvent_t e : c->prof_events) cudaEventDestroy(e);
+  c->prof_events.clear();
+  c->prof_used = 0;
+  return SDSAT_OK;
+}
+
 sdsat_status sdsat_build_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32_t* prev_out_dev,
                                const int32_t* prev_acc_dev, const int32_t* draft_table_dev, int table_stride,
                                int b, int q, int32_t* tokens_out_dev) {
@@ -551,8 +643,10 @@ sdsat_status sdsat_build_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32
   if ((mode != 1 && mode != 2) || b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q) return SDSAT_EINVAL;
   if (mode == 1 && c->cfg.n_adaptive > 1 && q - 1 > c->cfg.n_adaptive) return SDSAT_EINVAL;
   if (draft_table_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
-  return launch_build_block(mode, prev_out_dev, prev_acc_dev, draft_table_dev, table_stride, kv->len, c->adaptive,
-                            b, q, tokens_out_dev, c->stream, true) == cudaSuccess
+  return timed(c, K_BUILD_BLOCK, [&] {
+           return launch_build_block(mode, prev_out_dev, prev_acc_dev, draft_table_dev, table_stride, kv->len,
+                                     c->adaptive, b, q, tokens_out_dev, c->stream, true);
+         }) == cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;
 }
@@ -580,7 +674,8 @@ sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const
   g.epi = EPI_STORE;
   g.out = y_dev;
   g.out_ld = N;
-  return launch_gemm(g, c->num_sms, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+  return timed(c, K_GEMM_OP, [&] { return launch_gemm(g, c->num_sms, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+                                                                                                  : SDSAT_ECUDA;
 }
 
 sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_dev, const void* v_dev,
@@ -614,7 +709,8 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   a.nch_max = (cap + ATT_CHUNK - 1) / ATT_CHUNK;
   a.counters = c->att_counters;
   a.err = c->err;
-  return launch_attention(a, c->stream, true) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
+  return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+                                                                                                   : SDSAT_ECUDA;
 }
 
 sdsat_status sdsat_op_exp(sdsat_ctx* c, const float* in_dev, float* out_dev, int n) {
