@@ -186,7 +186,7 @@ class Runner:
         n_ref = 2 * self.new + 8 * self.q
         ref = torch.zeros(n_ref, self.b, dtype=torch.int32, device=self.dev)
         lg = torch.empty(self.b, self.shape.vocab, device=self.dev)
-        tok = self.init_out.view(self.b, self.q)[:, 0].contiguous()
+        tok = self.init_out.view(self.b, self.q)[:, 0].clone()   # a copy: init_out must stay intact
         acc = torch.empty(self.b, dtype=torch.int32, device=self.dev)
         wl = self.wl
         n_run = min(n_ref, self.cap - self.P)

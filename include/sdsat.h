@@ -254,6 +254,13 @@ SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, co
                                 const int32_t* len_dev, int b, int q, int H, int hd, int cap,
                                 float* out_dev);
 
+/* Copy a context workspace of the last block forward into dst_dev (fp32,
+ * rows x cols row-major, rows = b*q of that forward): which = 0 the residual
+ * stream h [rows][d], 1 the RoPE'd queries [rows][H*hd], 2 the attention
+ * output [rows][H*hd], 3 the SwiGLU activations [rows][F] -- of the last
+ * layer.  For tests that check a forward stage by stage.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_debug_workspace(sdsat_ctx* ctx, int which, int rows, float* dst_dev);
+
 /* out[i] = the nucleus sampler's exp (see sdsat_accept_nucleus) of in[i] <= 0. */
 SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* out_dev, int n);
 

@@ -90,6 +90,7 @@ def _lib():
             "sdsat_op_gemm": [P, P, I, I, P, I, P],
             "sdsat_op_attention": [P, P, P, P, P, I, I, I, I, I, P],
             "sdsat_op_exp": [P, P, P, I],
+            "sdsat_debug_workspace": [P, I, I, P],
         }
         for name, args in sig.items():
             fn = getattr(lib, name)
@@ -302,6 +303,16 @@ class Context:
         self._bind_stream()
         _check(_lib().sdsat_op_attention(self.handle, _ptr(q), _ptr(k), _ptr(v), _ptr(lens), b, qn, H, hd, cap,
                                          _ptr(out)), "sdsat_op_attention")
+
+    def debug_workspace(self, which: int, rows: int):
+        """Last-layer workspace of the last forward: 0 h, 1 q, 2 attention out, 3 SwiGLU act."""
+        import torch
+        s = self.shape
+        cols = [s.d_model, s.n_heads * s.head_dim, s.n_heads * s.head_dim, s.ffn_dim][which]
+        out = torch.empty(rows, cols, device="cuda")
+        self._bind_stream()
+        _check(_lib().sdsat_debug_workspace(self.handle, which, rows, _ptr(out)), "sdsat_debug_workspace")
+        return out
 
     def op_exp(self, x, y):
         self._bind_stream()

@@ -10,6 +10,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -77,6 +78,7 @@ struct sdsat_ctx {
   CUtensorMap head_map{};
   cudaStream_t stream = nullptr;
   int device = 0, num_sms = 0;
+  bool pdl = true;   // programmatic dependent launch between consecutive kernels
   // workspaces
   float2* rope = nullptr;
   float* h = nullptr;
@@ -180,7 +182,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
   const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
   if (timed(c, K_EMBED, [&] {
         return launch_embed(tokens, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, d, M, c->h, c->err,
-                            st, true);
+                            st, c->pdl);
       }) != cudaSuccess)
     return SDSAT_ECUDA;
   for (int l = 0; l < cf.n_layers; ++l) {
@@ -215,7 +217,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.positions = positions;
     g.rope = c->rope;
     g.rope_len = cf.max_position;
-    if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // block-causal attention
     AttnParams a;
     std::memset(&a, 0, sizeof(a));
@@ -237,7 +239,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
     a.counters = c->att_counters;
     a.err = c->err;
-    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // O projection + residual
     g = gemm_base(c, M);
     set_plain(g, mp.o, d, R);
@@ -246,7 +248,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
-    if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // gate/up with the fused RMSNorm and SiLU(gate) * up
     g = gemm_base(c, M);
     g.tmap[0] = mp.gate;
@@ -263,7 +265,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_SWIGLU;
     g.out = c->act;
     g.out_ld = F;
-    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // down projection + residual
     g = gemm_base(c, M);
     set_plain(g, mp.down, d, F);
@@ -272,7 +274,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
-    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
   }
   if (logits) {
     GemmParams g = gemm_base(c, M);
@@ -284,7 +286,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_STORE;
     g.out = logits;
     g.out_ld = cf.vocab;
-    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, true); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
   }
   return SDSAT_OK;
 }
@@ -321,7 +323,7 @@ sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, cons
   p.counters = c->acc_counters;
   p.err = c->err;
   p.emitted = kv->emitted;
-  return timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+  return timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, c->pdl); }) == cudaSuccess ? SDSAT_OK
                                                                                           : SDSAT_ECUDA;
 }
 
@@ -359,6 +361,10 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
   if (!c) return SDSAT_ENOMEM;
   c->cfg = *cfg;
   c->stream = static_cast<cudaStream_t>(stream);
+  {
+    const char* e = std::getenv("SDSAT_NO_PDL");   // e.g. for tools that cannot follow PDL launches
+    c->pdl = !(e && e[0] && e[0] != '0');
+  }
   if (cudaGetDevice(&c->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess ||
       gemm_prepare() != cudaSuccess) {
@@ -549,7 +555,7 @@ sdsat_status sdsat_prefill(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
     const int qn = std::min(SDSAT_MAX_Q, n - i);
     const sdsat_status s = forward(c, kv, seq, 1, qn, tokens_dev + i, nullptr, nullptr);
     if (s != SDSAT_OK) return s;
-    if (timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, true); }) !=
+    if (timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, c->pdl); }) !=
         cudaSuccess)
       return SDSAT_ECUDA;
   }
@@ -572,7 +578,7 @@ sdsat_status sdsat_accept_nucleus(sdsat_ctx* c, sdsat_kv* kv, const float* logit
 
 sdsat_status sdsat_kv_commit(sdsat_ctx* c, sdsat_kv* kv, const int32_t* new_len_dev, int b) {
   if (!c || !kv || kv->ctx != c || !new_len_dev || b < 1 || b > kv->batch || b > 64) return SDSAT_EINVAL;
-  return timed(c, K_KV_COMMIT, [&] { return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, true); }) ==
+  return timed(c, K_KV_COMMIT, [&] { return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, c->pdl); }) ==
                  cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;
@@ -645,7 +651,7 @@ sdsat_status sdsat_build_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32
   if (draft_table_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
   return timed(c, K_BUILD_BLOCK, [&] {
            return launch_build_block(mode, prev_out_dev, prev_acc_dev, draft_table_dev, table_stride, kv->len,
-                                     c->adaptive, b, q, tokens_out_dev, c->stream, true);
+                                     c->adaptive, b, q, tokens_out_dev, c->stream, c->pdl);
          }) == cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;
@@ -674,7 +680,7 @@ sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const
   g.epi = EPI_STORE;
   g.out = y_dev;
   g.out_ld = N;
-  return timed(c, K_GEMM_OP, [&] { return launch_gemm(g, c->num_sms, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+  return timed(c, K_GEMM_OP, [&] { return launch_gemm(g, c->num_sms, c->stream, c->pdl); }) == cudaSuccess ? SDSAT_OK
                                                                                                   : SDSAT_ECUDA;
 }
 
@@ -709,8 +715,19 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   a.nch_max = (cap + ATT_CHUNK - 1) / ATT_CHUNK;
   a.counters = c->att_counters;
   a.err = c->err;
-  return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->stream, true); }) == cudaSuccess ? SDSAT_OK
+  return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->stream, c->pdl); }) == cudaSuccess ? SDSAT_OK
                                                                                                    : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_debug_workspace(sdsat_ctx* c, int which, int rows, float* dst_dev) {
+  if (!c || !dst_dev || rows < 1 || rows > SDSAT_MAX_ROWS || which < 0 || which > 3) return SDSAT_EINVAL;
+  const int R = c->cfg.n_heads * c->cfg.head_dim;
+  const float* src[4] = {c->h, c->qbuf, c->attn, c->act};
+  const int cols[4] = {c->cfg.d_model, R, R, c->cfg.ffn_dim};
+  return cudaMemcpyAsync(dst_dev, src[which], (size_t)rows * cols[which] * sizeof(float), cudaMemcpyDeviceToDevice,
+                         c->stream) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
 }
 
 sdsat_status sdsat_op_exp(sdsat_ctx* c, const float* in_dev, float* out_dev, int n) {

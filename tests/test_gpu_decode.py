@@ -151,7 +151,9 @@ def test_tiny_device_loop_equals_plain_greedy(sd, tiny):
     out[0] = int(prompt[-1])
     toks = torch.empty(Q, dtype=torch.int32, device="cuda")
     emitted = []
+    per_loop = []
     while len(emitted) < N_NEW:
+        n_loop = 0
         for mode in (1, 2):
             ctx.build_block(kv, mode, out, acc, toks, 1, Q, draft_table=tab if mode == 2 else None,
                             table_stride=tab.numel())
@@ -159,6 +161,11 @@ def test_tiny_device_loop_equals_plain_greedy(sd, tiny):
             ctx.accept_greedy(kv, logits, toks, 1, Q, 0 if mode == 1 else K, acc, out)
             a = int(acc.item())
             emitted += out[:a].cpu().tolist()
+            n_loop += a
+        per_loop.append(n_loop)
+    # the stub drafts the true token with probability 0.7, so loops accept drafts (Sec. 2.1.1: 2..k+2 per loop)
+    assert all(2 <= n <= K + 2 for n in per_loop)
+    assert np.mean(per_loop) > 3.0, per_loop
     emitted = emitted[:N_NEW]
     same = sum(int(a == b) for a, b in zip(emitted, ref[:N_NEW]))
     first_diff = next((i for i, (a, b) in enumerate(zip(emitted, ref)) if a != b), None)
