@@ -325,7 +325,7 @@ def run_ours(args, wl, rank, world):
     # --- profiled pass (per-kernel CUDA events; launches serialised) for the roofline
     r.reset()
     n_prof = min(args.steps, steps_per_gen)
-    launches_per_step = 4 + 5 * shape.n_layers
+    launches_per_step = 4 + 7 * shape.n_layers   # build, norm, 7 per layer, head, accept
     r.ctx.profile_begin(n_prof * (launches_per_step + 2) + 16)
     r.run_steps(n_prof, steps_per_gen, None)
     kstats = r.ctx.profile_end()
@@ -541,6 +541,83 @@ def run_reference(args, wl, rank, world):
             "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# ----------------------------------------------------------------------------- kernel sweeps
+SWEEP_GEMM_SHAPES = [(4096, 12288), (4096, 22016), (11008, 4096), (4096, 32016)]   # (K, N): QKV, gate+up, down, head
+SWEEP_Q = [1, 2, 4, 6, 8, 11, 16]
+SWEEP_CTX = [512, 2048, 8192, 16384]
+
+
+def run_sweep(args):
+    """Kernel sweeps on 7B shapes (one JSON line per case): the skinny GEMM with M = q against
+    bf16 weights, and block-causal attention of q rows (32 heads x 128) against a bf16 cache.
+    Weights/caches rotate over enough buffers to exceed L2 between repetitions."""
+    import torch
+    import synth
+    import paper_2403_18647_gb300 as sd
+    torch.cuda.set_device(0)
+    peak, kind = peaks()
+    ctx = sd.Context(synth.SHAPES["7b"], None, max_position=16384 + 64)
+    reps = args.reps
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    cases = []
+    if args.sweep in ("gemm", "all"):
+        shapes = [tuple(int(v) for v in args.shape.split("x"))] if args.shape else SWEEP_GEMM_SHAPES
+        qs = [args.m] if args.m else SWEEP_Q
+        for K, N in shapes:
+            nbuf = max(2, int(math.ceil(4 * l2 / (K * N * 2))))
+            ws = [synth.normal_bf16(7, i, (N, K), 0.02, device="cuda") for i in range(nbuf)]
+            for M in qs:
+                x = synth.normal_f32(7, 100 + M, (M, K), 1.0, device="cuda")
+                y = torch.empty(M, N, device="cuda")
+                for i in range(3):
+                    ctx.op_gemm(x, ws[i % nbuf], y)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                for i in range(reps):
+                    ctx.op_gemm(x, ws[i % nbuf], y)
+                e1.record()
+                torch.cuda.synchronize()
+                us = e0.elapsed_time(e1) * 1e3 / reps
+                by = K * N * 2 + M * K * 4 + M * N * 4
+                cases.append({"kernel": "skinny_gemm", "M": M, "K": K, "N": N, "us": round(us, 2),
+                              "GB/s": round(by / us / 1e3, 1), "frac_of_measured": round(by / us / 1e3 / peak, 4),
+                              "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4),
+                              "note": "includes the fp32 -> bf16 hi/lo operand split kernel"})
+            del ws
+    if args.sweep in ("attention", "all"):
+        H, hd = 32, 128
+        ctxs = [args.ctx] if args.ctx else SWEEP_CTX
+        qs = [args.m] if args.m else SWEEP_Q
+        for n in ctxs:
+            cap = n + 16
+            nbuf = max(2, int(math.ceil(4 * l2 / (2 * H * cap * hd * 2))))
+            Ks = [synth.normal_bf16(8, 2 * i, (H * cap, hd), 1.0, device="cuda") for i in range(nbuf)]
+            Vs = [synth.normal_bf16(8, 2 * i + 1, (H * cap, hd), 1.0, device="cuda") for i in range(nbuf)]
+            ln = torch.tensor([n], dtype=torch.int32, device="cuda")
+            for q in qs:
+                Q = synth.normal_f32(8, 50 + q, (q, H * hd), 1.0, device="cuda")
+                out = torch.empty(q, H * hd, device="cuda")
+                for i in range(3):
+                    ctx.op_attention(Q, Ks[i % nbuf], Vs[i % nbuf], ln, 1, q, H, hd, cap, out)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                for i in range(reps):
+                    ctx.op_attention(Q, Ks[i % nbuf], Vs[i % nbuf], ln, 1, q, H, hd, cap, out)
+                e1.record()
+                torch.cuda.synchronize()
+                us = e0.elapsed_time(e1) * 1e3 / reps
+                by = 2 * H * (n + q) * hd * 2 + 2 * q * H * hd * 4
+                cases.append({"kernel": "attention", "q": q, "ctx": n, "heads": H, "head_dim": hd,
+                              "us": round(us, 2), "GB/s": round(by / us / 1e3, 1),
+                              "frac_of_measured": round(by / us / 1e3 / peak, 4),
+                              "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4)})
+            del Ks, Vs
+    for c in cases:
+        print(json.dumps(c), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -549,7 +626,15 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="7b", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", choices=["gemm", "attention", "all"], help="kernel sweeps instead of the step bench")
+    ap.add_argument("--shape", default="", help="sweep one GEMM shape KxN")
+    ap.add_argument("--m", type=int, default=0, help="sweep one M (GEMM) or q (attention)")
+    ap.add_argument("--ctx", type=int, default=0, help="sweep one attention context length")
+    ap.add_argument("--reps", type=int, default=50)
     args = ap.parse_args()
+    if args.sweep:
+        run_sweep(args)
+        return
     if args.warmup < 3:
         args.warmup = 3
     wl = WORKLOADS[args.config]

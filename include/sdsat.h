@@ -123,7 +123,7 @@ SDSAT_API sdsat_status sdsat_set_stream(sdsat_ctx* ctx, void* stream);
 /* Library-owned KV cache for `batch` sequences of up to `max_len` slots:
  * K and V bf16 [n_layers][batch][n_heads][max_len][head_dim], and the committed
  * length len[batch] (int32, device, starts at 0).  Synchronous.
- * Errors: EINVAL, ENOMEM. */
+ * Errors: EINVAL, ENOMEM, ECAPACITY (max_len > max_position or > 32768). */
 SDSAT_API sdsat_status sdsat_kv_create(sdsat_ctx* ctx, int batch, int max_len, sdsat_kv** out);
 SDSAT_API void sdsat_kv_destroy(sdsat_kv* kv);
 

@@ -396,26 +396,88 @@ cudaError_t launch_accept(const AcceptParams& p, cudaStream_t st, bool pdl) {
   return cudaLaunchKernelEx(&cfg, accept_kernel, p);
 }
 
-// ---- embedding gather: h[m][:] = E[token[m]][:] (fp32) ---------------------------------
-__global__ void embed_kernel(const int* tokens, const __nv_bfloat16* E, int V, int d, float* h, uint32_t* err) {
+// ---- RMSNorm into the GEMM operand ------------------------------------------------------
+// x = h * rsqrt(mean(h^2) + eps) * g (Llama's RMSNorm, fp32), stored as bf16 hi + lo with
+// hi = bf16(x), lo = bf16(x - hi), so hi + lo carries ~16 significant bits of x.  With
+// tokens != null the row is first gathered from the embedding table (h = E[token]).
+__device__ __forceinline__ void split_store(float v, __nv_bfloat16* hi, __nv_bfloat16* lo) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(v);
+  *hi = h;
+  *lo = __float2bfloat16_rn(v - __bfloat162float(h));
+}
+
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const int* tokens, const __nv_bfloat16* E, int V, float* h,
+                                                      int d, const __nv_bfloat16* g, float eps, __nv_bfloat16* xhi,
+                                                      __nv_bfloat16* xlo, uint32_t* err) {
+  __shared__ float red[32];
   pdl_wait();
   pdl_trigger();
   const int m = blockIdx.x;
-  int t = __ldcg(tokens + m);
-  if (t < 0 || t >= V) {
-    if (threadIdx.x == 0) set_error(err, ERR_TOKEN);
-    t = 0;
+  float* hr = h + (size_t)m * d;
+  const __nv_bfloat16* er = nullptr;
+  if (tokens) {
+    int t = __ldcg(tokens + m);
+    if (t < 0 || t >= V) {
+      if (threadIdx.x == 0) set_error(err, ERR_TOKEN);
+      t = 0;
+    }
+    er = E + (size_t)t * d;
   }
-  const __nv_bfloat162* src = reinterpret_cast<const __nv_bfloat162*>(E + (size_t)t * d);
-  float2* dst = reinterpret_cast<float2*>(h + (size_t)m * d);
-  for (int i = threadIdx.x; i < d / 2; i += blockDim.x) dst[i] = __bfloat1622float2(src[i]);
+  float ss = 0.f;
+  for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
+    float4 v;
+    if (er) {
+      const __nv_bfloat162* e2 = reinterpret_cast<const __nv_bfloat162*>(er + i);
+      const float2 a = __bfloat1622float2(e2[0]), b = __bfloat1622float2(e2[1]);
+      v = make_float4(a.x, a.y, b.x, b.y);
+      *reinterpret_cast<float4*>(hr + i) = v;
+    } else {
+      v = __ldcg(reinterpret_cast<const float4*>(hr + i));
+    }
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float t = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) red[0] = t;
+  }
+  __syncthreads();
+  const float inv = 1.0f / sqrtf(red[0] / (float)d + eps);
+  for (int i = threadIdx.x * 4; i < d; i += blockDim.x * 4) {
+    const float4 v = __ldcg(reinterpret_cast<const float4*>(hr + i));
+    const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      split_store(vv[e] * inv * __bfloat162float(g[i + e]), xhi + (size_t)m * d + i + e, xlo + (size_t)m * d + i + e);
+  }
 }
 
-cudaError_t launch_embed(const int* tokens, const __nv_bfloat16* E, int V, int d, int M, float* h,
-                         uint32_t* err, cudaStream_t st, bool pdl) {
+cudaError_t launch_rmsnorm(const int* tokens, const __nv_bfloat16* E, int V, float* h, int d, int M,
+                           const __nv_bfloat16* gain, float eps, __nv_bfloat16* xhi, __nv_bfloat16* xlo,
+                           uint32_t* err, cudaStream_t st, bool pdl) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(M), dim3(256), st, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, embed_kernel, tokens, E, V, d, h, err);
+  return cudaLaunchKernelEx(&cfg, rmsnorm_kernel, tokens, E, V, h, d, gain, eps, xhi, xlo, err);
+}
+
+__global__ void split_kernel(const float* x, int n, __nv_bfloat16* xhi, __nv_bfloat16* xlo) {
+  pdl_wait();
+  pdl_trigger();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) split_store(__ldcg(x + i), xhi + i, xlo + i);
+}
+
+cudaError_t launch_split(const float* x, int M, int K, __nv_bfloat16* xhi, __nv_bfloat16* xlo, cudaStream_t st,
+                         bool pdl) {
+  cudaLaunchAttribute attr[1];
+  const int n = M * K;
+  cudaLaunchConfig_t cfg = make_cfg(dim3((n + 255) / 256), dim3(256), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, split_kernel, x, n, xhi, xlo);
 }
 
 // ---- block input of draft step 1 (mode 1) and draft step 2 (mode 2) --------------------

@@ -7,119 +7,273 @@
 // hd*2 bytes each), read once per (sequence, head) for all q rows together.
 //
 // Grid (chunk, head, sequence): each CTA owns ATT_CHUNK = 128 consecutive
-// slots, computes for every block row the chunk's max score, exp-sum and
-// unnormalised output, and writes them to a workspace; the last CTA of a
-// (sequence, head) (per-pair counter, no waiting) merges the chunks in chunk
-// order with the usual log-sum-exp rescaling -- deterministic.
+// slots.  One thread issues TMA loads of the chunk's K and V tiles (boxes of
+// 64 dims x 128 rows, 128-byte swizzle) as soon as the previous kernel has
+// finished; K and V land on separate mbarriers so the scores are computed
+// while V is still in flight.  Both products run on the tensor cores
+// (mma.sync m16n8k16, the q <= 16 rows fill the M = 16 tile): S = Q K^T with
+// each warp on 32 keys, then O = P V with each warp on hd/4 dimensions.  Q
+// and P enter as bf16 hi + lo pairs (two MMAs each), K and V are the cache's
+// own bf16 values, accumulation is fp32.  Each CTA
+// writes its chunk's max score, exp-sum and unnormalised output per row; the
+// last CTA of a (sequence, head) (per-pair counter, no waiting) merges the
+// chunks in chunk order with the usual log-sum-exp rescaling --
+// deterministic -- and writes the output in fp32 and as the O projection's
+// bf16 hi + lo operand.
 #include "common.cuh"
 #include "internal.h"
 
 namespace sdsat {
 
 template <int HD>
-__global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
-  constexpr int CH = ATT_CHUNK;
-  __shared__ __align__(16) float Qs[SDSAT_ATT_MAXQ][HD];
-  __shared__ float Ps[SDSAT_ATT_MAXQ][CH];
-  __shared__ float Ms[SDSAT_ATT_MAXQ], Ls[SDSAT_ATT_MAXQ];
-  __shared__ int s_last;
+struct AttCfg {
+  static constexpr int HALVES = HD / 64;                 // 64-dim column boxes per row
+  static constexpr int TILE = ATT_CHUNK * 128 * HALVES;  // bytes of one K (or V) chunk
+  static constexpr int QSTRIDE = HD * 2 + 16;            // bytes per row of the bf16 Q / P tiles (padded)
+  static constexpr int PSTRIDE = ATT_CHUNK * 2 + 16;
+  static constexpr size_t SMEM = 1024 + 2 * (size_t)TILE + 2 * 16 * QSTRIDE + 2 * 16 * PSTRIDE +
+                                 2 * 4 * 16 * 4 + 2 * 16 * 4 + 64;
+};
 
-  pdl_wait();
-  pdl_trigger();
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo_elem, float hi_elem) {
+  return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(lo_elem)) |
+         ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi_elem)) << 16);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ AttnParams p) {
+  using C = AttCfg<HD>;
+  constexpr int CH = ATT_CHUNK;
+  constexpr int KSTEPS = HD / 16;          // MMA k-steps over the head dimension
+  constexpr int DT = HD / 32;              // 8-wide dimension tiles per warp in P.V
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Ktile = smem;
+  uint8_t* Vtile = smem + C::TILE;
+  uint8_t* Qh = smem + 2 * C::TILE;                 // bf16 [16][HD] (scaled q, hi part), padded rows
+  uint8_t* Ql = Qh + 16 * C::QSTRIDE;               // lo part
+  uint8_t* Ph = Ql + 16 * C::QSTRIDE;               // bf16 [16][CH] softmax numerators, hi part
+  uint8_t* Pl = Ph + 16 * C::PSTRIDE;
+  float* red_m = reinterpret_cast<float*>(Pl + 16 * C::PSTRIDE);   // [4 warps][16 rows]
+  float* red_l = red_m + 64;
+  float* Ms = red_l + 64;                           // [16] chunk max per row
+  float* Ls = Ms + 16;                              // [16] chunk exp-sum per row
+  uint64_t* bar = reinterpret_cast<uint64_t*>(Ls + 16);   // [0] K landed, [1] V landed
+  int* s_last = reinterpret_cast<int*>(bar + 2);
+
   const int ch = blockIdx.x, h = blockIdx.y, sl = blockIdx.z, s = p.seq0 + sl;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, tig = lane & 3;
   const int q = p.q;
+  pdl_trigger();
+  // The committed length is final before this kernel can start: the block forward's
+  // first kernel (RMSNorm) lets its dependents launch only after every earlier kernel
+  // has completed.  Slots below it are not written during this forward either, so a
+  // chunk that lies entirely below it can be loaded before the QKV projection finishes.
   const int len = __ldcg(p.len + s);
   const int nkeys = min(len + q, p.cap);
   const int c0 = ch * CH;
   if (c0 >= nkeys) return;
   const int nch = (nkeys + CH - 1) / CH;
-  const float scale = rsqrtf((float)HD);
-
-  for (int i = tid; i < q * HD; i += 128) {
-    const int j = i / HD, d = i % HD;
-    Qs[j][d] = __ldcg(p.Q + (size_t)(sl * q + j) * p.q_ld + h * HD + d) * scale;
+  const int row0 = p.row0 + (s * p.H + h) * p.cap + c0;   // first cache row of the chunk
+  const bool early = c0 + CH <= len;                        // chunk holds committed slots only
+  uint64_t pol = 0;
+  auto issue_loads = [&]() {
+    mbar_arrive_expect_tx(&bar[0], C::TILE);
+#pragma unroll
+    for (int hh = 0; hh < C::HALVES; ++hh) tma_load_2d(Ktile + hh * CH * 128, &p.kmap, &bar[0], hh * 64, row0, pol);
+    mbar_arrive_expect_tx(&bar[1], C::TILE);
+#pragma unroll
+    for (int hh = 0; hh < C::HALVES; ++hh) tma_load_2d(Vtile + hh * CH * 128, &p.vmap, &bar[1], hh * 64, row0, pol);
+  };
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_mbar_init();
+    pol = l2_policy_evict_first();
+    if (early) issue_loads();
   }
-  __syncthreads();
+  pdl_wait();   // q and this forward's new K/V rows come from the QKV projection
+  if (tid == 0 && !early) issue_loads();
+  // q (scaled by 1/sqrt(hd)) as bf16 hi + lo; rows >= q are zero
+  const float scale = rsqrtf((float)HD);
+  for (int i = tid; i < 16 * (HD / 2); i += 128) {
+    const int j = i / (HD / 2), d = (i % (HD / 2)) * 2;
+    float x0 = 0.f, x1 = 0.f;
+    if (j < q) {
+      const float2 v = __ldcg(reinterpret_cast<const float2*>(p.Q + (size_t)(sl * q + j) * p.q_ld + h * HD + d));
+      x0 = v.x * scale;
+      x1 = v.y * scale;
+    }
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+    *reinterpret_cast<uint32_t*>(Qh + j * C::QSTRIDE + d * 2) =
+        (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    *reinterpret_cast<uint32_t*>(Ql + j * C::QSTRIDE + d * 2) =
+        pack_bf16(x0 - __bfloat162float(h0), x1 - __bfloat162float(h1));
+  }
+  __syncthreads();   // Q tiles and the barrier initialisation are visible to all threads
 
-  // scores: thread t <-> slot c0 + t
-  const size_t head_base = ((size_t)s * p.H + h) * p.cap;
-  {
-    const int kp = c0 + tid;
-    float sc[SDSAT_ATT_MAXQ];
+  volatile int no_abort = 0;
+  bool ok = mbar_wait_bounded(&bar[0], 0, &no_abort, p.err);
+
+  // ---- S = Q K^T for this warp's 32 keys (4 tiles of 8), fp32 in registers
+  const int kb = warp * 32;                       // first key (within the chunk) of this warp
+  float S[4][4];
 #pragma unroll
-    for (int j = 0; j < SDSAT_ATT_MAXQ; ++j) sc[j] = 0.f;
-    if (kp < nkeys) {
-      const uint4* kr = reinterpret_cast<const uint4*>(p.k + (head_base + kp) * HD);
-#pragma unroll 4
-      for (int gi = 0; gi < HD / 8; ++gi) {
-        const uint4 raw = __ldcg(kr + gi);
-        const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-        float kf[8];
+  for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __bfloat1622float2(k2[e]);
-          kf[2 * e] = f.x;
-          kf[2 * e + 1] = f.y;
-        }
+    for (int e = 0; e < 4; ++e) S[nt][e] = 0.f;
+  const int mi = lane >> 3, r8 = lane & 7;        // ldmatrix: this thread's matrix and row
+  if (ok) {
 #pragma unroll
-        for (int j = 0; j < SDSAT_ATT_MAXQ; ++j) {
-          if (j < q) {
-            const float4 a = *reinterpret_cast<const float4*>(&Qs[j][gi * 8]);
-            const float4 b = *reinterpret_cast<const float4*>(&Qs[j][gi * 8 + 4]);
-            sc[j] += a.x * kf[0] + a.y * kf[1] + a.z * kf[2] + a.w * kf[3] + b.x * kf[4] + b.y * kf[5] +
-                     b.z * kf[6] + b.w * kf[7];
-          }
-        }
+    for (int kk = 0; kk < KSTEPS; ++kk) {
+      uint32_t ah[4], al[4];
+      const int qrow = r8 + 8 * (mi & 1), qcol = kk * 16 + 8 * (mi >> 1);
+      ldsm_x4(smem_u32(Qh + qrow * C::QSTRIDE + qcol * 2), ah[0], ah[1], ah[2], ah[3]);
+      ldsm_x4(smem_u32(Ql + qrow * C::QSTRIDE + qcol * 2), al[0], al[1], al[2], al[3]);
+      const int hh = kk >> 2, cg = 2 * (kk & 3);  // 64-dim half and first 16-byte granule
+#pragma unroll
+      for (int np = 0; np < 2; ++np) {            // two key tiles per ldmatrix.x4
+        const int key = kb + 8 * (2 * np + (mi >> 1)) + r8;
+        const int c = cg + (mi & 1);
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(smem_u32(Ktile + hh * CH * 128 + key * 128 + ((c ^ (key & 7)) << 4)), b0, b1, b2, b3);
+        mma_bf16_16816(S[2 * np], ah[0], ah[1], ah[2], ah[3], b0, b1);
+        mma_bf16_16816(S[2 * np], al[0], al[1], al[2], al[3], b0, b1);
+        mma_bf16_16816(S[2 * np + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+        mma_bf16_16816(S[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
       }
     }
+  }
+  // mask: row j sees chunk key k iff c0 + k <= len + j (and c0 + k < nkeys, j < q)
 #pragma unroll
-    for (int j = 0; j < SDSAT_ATT_MAXQ; ++j)
-      if (j < q) Ps[j][tid] = (kp < nkeys && kp <= len + j) ? sc[j] : -INFINITY;
+  for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = g + 8 * (e >> 1);
+      const int kp = c0 + kb + 8 * nt + 2 * tig + (e & 1);
+      if (!ok || j >= q || kp >= nkeys || kp > len + j) S[nt][e] = -INFINITY;
+    }
+  // ---- row max and exp-sum over the chunk's 128 keys (4 threads x 4 warps share a row)
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int nt = 0; nt < 4; ++nt) {
+    mx0 = fmaxf(mx0, fmaxf(S[nt][0], S[nt][1]));
+    mx1 = fmaxf(mx1, fmaxf(S[nt][2], S[nt][3]));
+  }
+#pragma unroll
+  for (int o = 1; o < 4; o <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+  }
+  if (tig == 0) {
+    red_m[warp * 16 + g] = mx0;
+    red_m[warp * 16 + g + 8] = mx1;
   }
   __syncthreads();
-
-  // per-row max and exp-sum over the chunk: warp w takes rows w, w+4, ...
-  for (int j = warp; j < q; j += 4) {
-    float m = -INFINITY;
-    for (int t = lane; t < CH; t += 32) m = fmaxf(m, Ps[j][t]);
+  mx0 = fmaxf(fmaxf(red_m[g], red_m[16 + g]), fmaxf(red_m[32 + g], red_m[48 + g]));
+  mx1 = fmaxf(fmaxf(red_m[8 + g], red_m[24 + g]), fmaxf(red_m[40 + g], red_m[56 + g]));
+  float l0 = 0.f, l1 = 0.f;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    float l = 0.f;
-    for (int t = lane; t < CH; t += 32) {
-      const float e = (m == -INFINITY) ? 0.f : expf(Ps[j][t] - m);
-      Ps[j][t] = e;
-      l += e;
+  for (int nt = 0; nt < 4; ++nt) {
+    float pv[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float m = (e < 2) ? mx0 : mx1;
+      pv[e] = (S[nt][e] == -INFINITY) ? 0.f : expf(S[nt][e] - m);
     }
+    l0 += pv[0] + pv[1];
+    l1 += pv[2] + pv[3];
+    const int key = kb + 8 * nt + 2 * tig;
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(pv[0]), h1 = __float2bfloat16_rn(pv[1]);
+    const __nv_bfloat16 h2 = __float2bfloat16_rn(pv[2]), h3 = __float2bfloat16_rn(pv[3]);
+    *reinterpret_cast<uint32_t*>(Ph + g * C::PSTRIDE + key * 2) =
+        (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    *reinterpret_cast<uint32_t*>(Ph + (g + 8) * C::PSTRIDE + key * 2) =
+        (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
+    *reinterpret_cast<uint32_t*>(Pl + g * C::PSTRIDE + key * 2) =
+        pack_bf16(pv[0] - __bfloat162float(h0), pv[1] - __bfloat162float(h1));
+    *reinterpret_cast<uint32_t*>(Pl + (g + 8) * C::PSTRIDE + key * 2) =
+        pack_bf16(pv[2] - __bfloat162float(h2), pv[3] - __bfloat162float(h3));
+  }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-    if (lane == 0) {
-      Ms[j] = m;
-      Ls[j] = l;
+  for (int o = 1; o < 4; o <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+  }
+  if (tig == 0) {
+    red_l[warp * 16 + g] = l0;
+    red_l[warp * 16 + g + 8] = l1;
+  }
+  __syncthreads();   // P tiles and the partial sums are complete
+  if (tid < 16) {
+    Ms[tid] = fmaxf(fmaxf(red_m[tid], red_m[16 + tid]), fmaxf(red_m[32 + tid], red_m[48 + tid]));
+    Ls[tid] = red_l[tid] + red_l[16 + tid] + red_l[32 + tid] + red_l[48 + tid];
+  }
+
+  // ---- O = P V for this warp's HD/4 dimensions (DT tiles of 8), all 128 keys
+  ok = ok && mbar_wait_bounded(&bar[1], 0, &no_abort, p.err);
+  float O[DT][4];
+#pragma unroll
+  for (int nt = 0; nt < DT; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) O[nt][e] = 0.f;
+  const int db = warp * (HD / 4);                 // first dimension of this warp
+  if (ok) {
+#pragma unroll
+    for (int kk = 0; kk < CH / 16; ++kk) {
+      uint32_t ah[4], al[4];
+      const int prow = r8 + 8 * (mi & 1), pcol = kk * 16 + 8 * (mi >> 1);
+      ldsm_x4(smem_u32(Ph + prow * C::PSTRIDE + pcol * 2), ah[0], ah[1], ah[2], ah[3]);
+      ldsm_x4(smem_u32(Pl + prow * C::PSTRIDE + pcol * 2), al[0], al[1], al[2], al[3]);
+#pragma unroll
+      for (int np = 0; np < DT / 2; ++np) {       // two dimension tiles per ldmatrix.x4.trans
+        const int key = kk * 16 + 8 * (mi & 1) + r8;
+        const int dim = db + 8 * (2 * np + (mi >> 1));
+        const int hh = dim >> 6, c = (dim & 63) >> 3;
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(smem_u32(Vtile + hh * CH * 128 + key * 128 + ((c ^ (key & 7)) << 4)), b0, b1, b2, b3);
+        mma_bf16_16816(O[2 * np], ah[0], ah[1], ah[2], ah[3], b0, b1);
+        mma_bf16_16816(O[2 * np], al[0], al[1], al[2], al[3], b0, b1);
+        mma_bf16_16816(O[2 * np + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+        mma_bf16_16816(O[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
+      }
     }
   }
-  __syncthreads();
-
-  // unnormalised output of the chunk: thread d <-> dimension d
-  const int nk = min(CH, nkeys - c0);
-  const size_t prow = (size_t)h * p.nch_max + ch;
-  if (tid < HD) {
-    float o[SDSAT_ATT_MAXQ];
+  const size_t prow_base = (size_t)h * p.nch_max + ch;
 #pragma unroll
-    for (int j = 0; j < SDSAT_ATT_MAXQ; ++j) o[j] = 0.f;
-    const __nv_bfloat16* vcol = p.v + head_base * HD + (size_t)c0 * HD + tid;
-    for (int t = 0; t < nk; ++t) {
-      const float v = __bfloat162float(vcol[(size_t)t * HD]);
+  for (int nt = 0; nt < DT; ++nt)
 #pragma unroll
-      for (int j = 0; j < SDSAT_ATT_MAXQ; ++j)
-        if (j < q) o[j] += Ps[j][t] * v;
+    for (int e = 0; e < 4; e += 2) {
+      const int j = g + 8 * (e >> 1);
+      if (j < q) {
+        const int dim = db + 8 * nt + 2 * tig;
+        *reinterpret_cast<float2*>(p.part_o + ((size_t)(sl * q + j) * p.H * p.nch_max + prow_base) * HD + dim) =
+            make_float2(O[nt][e], O[nt][e + 1]);
+      }
     }
-#pragma unroll
-    for (int j = 0; j < SDSAT_ATT_MAXQ; ++j)
-      if (j < q) p.part_o[((size_t)(sl * q + j) * p.H * p.nch_max + prow) * HD + tid] = o[j];
-  }
+  __syncthreads();   // Ms / Ls written
   if (tid < q) {
-    float* ml = p.part_ml + ((size_t)(sl * q + tid) * p.H * p.nch_max + prow) * 2;
+    float* ml = p.part_ml + ((size_t)(sl * q + tid) * p.H * p.nch_max + prow_base) * 2;
     ml[0] = Ms[tid];
     ml[1] = Ls[tid];
   }
@@ -127,33 +281,74 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
   // the last chunk CTA of this (sequence, head) merges the chunks
   __threadfence();
   __syncthreads();
-  if (tid == 0) s_last = (atomicAdd(p.counters + sl * p.H + h, 1) == nch - 1);
+  if (tid == 0) *s_last = (atomicAdd(p.counters + sl * p.H + h, 1) == nch - 1);
   __syncthreads();
-  if (!s_last) return;
+  if (!*s_last) return;
   __threadfence();
+  // chunk statistics of every row -> shared memory (the K tile is free now), then the
+  // per-row rescaling weights w[j][c] = exp(m_c - max_c m_c) and the normaliser L_j
+  float* w = reinterpret_cast<float*>(Ktile);          // [q][nch]; q*nch <= 16 * ATT_MAX_CHUNKS
+  float* lsum = w + q * nch;                            // [q][nch]; both fit the K + V tiles
+  for (int i = tid; i < q * nch; i += 128) {
+    const int j = i / nch, c = i % nch;
+    const float* ml = p.part_ml + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max + c) * 2;
+    w[i] = __ldcg(ml);
+    lsum[i] = __ldcg(ml + 1);
+  }
+  __syncthreads();
+  if (tid < q) {
+    float mx = -INFINITY;
+    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, w[tid * nch + c]);
+    float L = 0.f;
+    for (int c = 0; c < nch; ++c) {
+      const float mc = w[tid * nch + c];
+      const float wc = (mc == -INFINITY) ? 0.f : expf(mc - mx);
+      w[tid * nch + c] = wc;
+      L += wc * lsum[tid * nch + c];
+    }
+    Ms[tid] = 1.0f / L;
+  }
+  __syncthreads();
   if (tid < HD) {
     for (int j = 0; j < q; ++j) {
-      const size_t rb = (size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max;
-      float mx = -INFINITY;
-      for (int c = 0; c < nch; ++c) mx = fmaxf(mx, __ldcg(p.part_ml + (rb + c) * 2));
-      float L = 0.f, O = 0.f;
-      for (int c = 0; c < nch; ++c) {
-        const float mc = __ldcg(p.part_ml + (rb + c) * 2);
-        const float w = (mc == -INFINITY) ? 0.f : expf(mc - mx);
-        L += w * __ldcg(p.part_ml + (rb + c) * 2 + 1);
-        O += w * __ldcg(p.part_o + (rb + c) * HD + tid);
+      const float* po = p.part_o + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max) * HD + tid;
+      float O = 0.f;
+      int c = 0;
+      for (; c + 4 <= nch; c += 4) {   // four independent loads in flight
+        const float o0 = __ldcg(po + (size_t)c * HD), o1 = __ldcg(po + (size_t)(c + 1) * HD);
+        const float o2 = __ldcg(po + (size_t)(c + 2) * HD), o3 = __ldcg(po + (size_t)(c + 3) * HD);
+        O += w[j * nch + c] * o0;
+        O += w[j * nch + c + 1] * o1;
+        O += w[j * nch + c + 2] * o2;
+        O += w[j * nch + c + 3] * o3;
       }
-      p.out[(size_t)(sl * q + j) * p.out_ld + h * HD + tid] = O / L;
+      for (; c < nch; ++c) O += w[j * nch + c] * __ldcg(po + (size_t)c * HD);
+      const float o = O * Ms[j];
+      const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + tid;
+      p.out[idx] = o;
+      const __nv_bfloat16 hi = __float2bfloat16_rn(o);
+      p.out_hi[idx] = hi;
+      p.out_lo[idx] = __float2bfloat16_rn(o - __bfloat162float(hi));
     }
   }
   if (tid == 0) p.counters[sl * p.H + h] = 0;
+}
+
+size_t attention_smem_bytes(int hd) { return hd == 64 ? AttCfg<64>::SMEM : AttCfg<128>::SMEM; }
+
+cudaError_t attention_prepare() {
+  cudaError_t e = cudaFuncSetAttribute(attention_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)AttCfg<64>::SMEM);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attention_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)AttCfg<128>::SMEM);
 }
 
 cudaError_t launch_attention(const AttnParams& p, cudaStream_t st, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.nch_max, p.H, p.nb);
   cfg.blockDim = dim3(128);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = attention_smem_bytes(p.hd);
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -15,14 +15,18 @@
 //    into a ring of shared-memory stages; it needs nothing from the previous
 //    kernel, so with programmatic dependent launch it starts prefetching while
 //    the previous kernel drains.
-//  * Warps 2-3 build the activation operand per chunk: fp32 rows (optionally
-//    RMS-normalised with the gain, fusing the RMSNorm) split into bf16 hi + lo
-//    parts so that the tensor-core product keeps ~16 mantissa bits of X.
-//  * Warp 1 (one thread) issues tcgen05.mma: D[128 x MPAD] (fp32, TMEM) +=
-//    Wtile[128 x 16] * Xhi^T + Wtile * Xlo^T, four K-steps per chunk.  Two TMEM
+//    The activation operand X arrives the same way, once the previous kernel
+//    has finished: its producer (RMSNorm, attention merge, SwiGLU epilogue)
+//    stored it as two bf16 matrices hi + lo with x ~= hi + lo to ~16 mantissa
+//    bits, so the tensor-core product keeps fp32-like accuracy in X.
+//  * Warp 1 (one thread) issues tcgen05.mma: D[128 x 2*MPAD] (fp32, TMEM) +=
+//    Wtile[128 x 16] * [Xhi; Xlo]^T -- the hi and lo operands sit back to back
+//    in shared memory, so one MMA with N = 2*MPAD covers both and the epilogue
+//    adds column m and column MPAD + m.  Four K-steps per chunk.  Two TMEM
 //    accumulators alternate so a tile's epilogue overlaps the next tile's MMAs.
-//  * Warps 4-7 read the accumulator (tcgen05.ld) and run the fused epilogue:
-//    plain store, residual add, RoPE + KV-cache append, or SiLU(gate) * up.
+//  * Warps 2-5 read the accumulator (tcgen05.ld) and run the fused epilogue:
+//    plain store, residual add, RoPE + KV-cache append, or SiLU(gate) * up
+//    (which also emits the next GEMM's hi/lo operand).
 #include <algorithm>
 
 #include "common.cuh"
@@ -30,16 +34,28 @@
 
 namespace sdsat {
 
+// Pipeline depth and CTAs per SM (compile-time tuning).  Measured on GB300: one CTA
+// per SM streams ~5 TB/s whatever its depth (3..10 stages), two CTAs per SM ~7 TB/s.
+// For M <= 16 two 3-stage CTAs (~71 KB of shared memory each) run per SM, which
+// still leaves room for one CTA of the next kernel to start prefetching its weights.
+#ifndef SDSAT_GEMM_STAGES16
+#define SDSAT_GEMM_STAGES16 3
+#endif
+#ifndef SDSAT_GEMM_CTAS_PER_SM
+#define SDSAT_GEMM_CTAS_PER_SM 2
+#endif
+
 template <int MPAD>
 struct GemmCfg {
-  static constexpr int STAGES = MPAD <= 16 ? 5 : (MPAD <= 32 ? 4 : 3);
+  static constexpr int STAGES = MPAD <= 16 ? SDSAT_GEMM_STAGES16 : (MPAD <= 32 ? 4 : 3);
   static constexpr int W_BYTES = 128 * 128;      // 128 rows x 64 bf16
   static constexpr int X_BYTES = MPAD * 128;     // MPAD rows x 64 bf16 (hi or lo)
   static constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
   static constexpr int STAGING = 128 * (MPAD + 1);
-  static constexpr int TMEM_COLS = 2 * MPAD < 32 ? 32 : 2 * MPAD;
-  static constexpr int NBAR = 3 * STAGES + 5;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 64 * 4 + NBAR * 8 + 32;
+  static constexpr int ACC_COLS = 2 * MPAD;     // hi and lo products side by side
+  static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
+  static constexpr int NBAR = 2 * STAGES + 5;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + NBAR * 8 + 32;
 };
 
 __device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
@@ -98,7 +114,11 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
         if (m >= M) break;
         const float g = acc[m];
         const float u = staging[(r + 64) * (MPAD + 1) + m];
-        p.out[(size_t)m * p.out_ld + j] = g / (1.0f + expf(-g)) * u;
+        const float a = g / (1.0f + expf(-g)) * u;
+        p.out[(size_t)m * p.out_ld + j] = a;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(a);
+        p.out_hi[(size_t)m * p.out_ld + j] = hi;
+        p.out_lo[(size_t)m * p.out_ld + j] = __float2bfloat16_rn(a - __bfloat162float(hi));
       }
     }
   } else {  // EPI_QKV
@@ -140,19 +160,17 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
 }
 
 template <int MPAD>
-__global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ GemmParams p) {
+__global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ GemmParams p) {
   using C = GemmCfg<MPAD>;
   constexpr int S = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;
   float* staging = reinterpret_cast<float*>(smem + (size_t)S * C::STAGE_BYTES);
-  float* inv_rms = staging + C::STAGING;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(inv_rms + 64);
-  uint64_t* full = bars;             // weights landed (TMA)
-  uint64_t* xfull = bars + S;        // activation operand written
-  uint64_t* empty = bars + 2 * S;    // stage consumed by the tensor core
-  uint64_t* acc_full = bars + 3 * S; // [2] accumulator ready
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + C::STAGING);
+  uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
+  uint64_t* empty = bars + S;        // stage consumed by the tensor core
+  uint64_t* acc_full = bars + 2 * S; // [2] accumulator ready
   uint64_t* acc_empty = acc_full + 2;// [2] accumulator drained
   uint64_t* drain = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -167,7 +185,6 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&xfull[s], 2);
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -186,25 +203,48 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
   pdl_trigger();
 
   if (warp == 0) {
-    // ------------------------------------------------ weight stream (TMA)
+    // ------------------------------------------------ weight + activation stream (TMA)
     if (lane == 0) {
       const int nmaps = p.map_mode == MAP_QKV3 ? 3 : (p.map_mode == MAP_GATEUP ? 2 : 1);
       for (int i = 0; i < nmaps; ++i) tma_prefetch_desc(&p.tmap[i]);
-      const uint64_t pol = l2_policy_evict_first();
-      int it = 0;
-      for (long long g = g0; g < g1; ++g, ++it) {
-        const int s = it % S;
-        const uint32_t ph = (it / S) & 1;
-        if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, p.err)) break;
+      tma_prefetch_desc(&p.tmap_x[0]);
+      tma_prefetch_desc(&p.tmap_x[1]);
+      const uint64_t pol_w = l2_policy_evict_first();   // weights: read once per step
+      const uint64_t pol_x = l2_policy_evict_last();    // activations: read by every CTA
+      constexpr uint32_t TX = C::W_BYTES + 2 * C::X_BYTES;
+      const long long n = g1 - g0;
+      const int npre = (int)std::min<long long>(S, n);
+      auto load_w = [&](int it) {
+        const long long g = g0 + it;
         const int tile = (int)(g / p.kc), kc = (int)(g % p.kc);
-        uint8_t* dst = stages + (size_t)s * C::STAGE_BYTES;
-        mbar_arrive_expect_tx(&full[s], C::W_BYTES);
+        uint8_t* dst = stages + (size_t)(it % S) * C::STAGE_BYTES;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           int map, row;
           tile_half_src(p, tile, h, map, row);
-          tma_load_2d(dst + h * 8192, &p.tmap[map], &full[s], kc * 64, row, pol);
+          tma_load_2d(dst + h * 8192, &p.tmap[map], &full[it % S], kc * 64, row, pol_w);
         }
+      };
+      auto load_x = [&](int it) {
+        const int kc = (int)((g0 + it) % p.kc);
+        uint8_t* dst = stages + (size_t)(it % S) * C::STAGE_BYTES + C::W_BYTES;
+        tma_load_2d(dst, &p.tmap_x[0], &full[it % S], kc * 64, 0, pol_x);
+        tma_load_2d(dst + C::X_BYTES, &p.tmap_x[1], &full[it % S], kc * 64, 0, pol_x);
+      };
+      // weights of the first stages do not depend on the previous kernel: issue them now
+      for (int it = 0; it < npre; ++it) {
+        mbar_arrive_expect_tx(&full[it], TX);
+        load_w(it);
+      }
+      pdl_wait();   // the activations are the previous kernel's output
+      for (int it = 0; it < npre; ++it) load_x(it);
+      int it = npre;
+      for (; it < n; ++it) {
+        const int s = it % S;
+        if (!mbar_wait_bounded(&empty[s], ((it / S) & 1) ^ 1, abort_flag, p.err)) break;
+        mbar_arrive_expect_tx(&full[s], TX);
+        load_w(it);
+        load_x(it);
       }
       if (*abort_flag) {  // let every copy in flight land before the CTA exits
         for (int i = std::max(0, it - S); i < it; ++i) mbar_wait_drain(&full[i % S], (i / S) & 1);
@@ -213,7 +253,7 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
   } else if (warp == 1) {
     // ------------------------------------------------ tensor-core issue
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(128, MPAD);
+      constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * MPAD);
       int it = 0, seg = 0;
       long long g = g0;
       bool ok = true;
@@ -223,25 +263,21 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
         const int buf = seg & 1;
         if (!mbar_wait_bounded(&acc_empty[buf], ((seg >> 1) & 1) ^ 1, abort_flag, p.err)) break;
         tc_fence_after();
-        const uint32_t d = tmem + buf * MPAD;
+        const uint32_t d = tmem + buf * C::ACC_COLS;
         const long long gstart = g;
         for (; g < gend; ++g, ++it) {
           const int s = it % S;
           const uint32_t ph = (it / S) & 1;
-          if (!mbar_wait_bounded(&full[s], ph, abort_flag, p.err) ||
-              !mbar_wait_bounded(&xfull[s], ph, abort_flag, p.err)) {
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag, p.err)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t wa = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
-          const uint32_t xh = wa + C::W_BYTES, xl = xh + C::X_BYTES;
+          const uint32_t xh = wa + C::W_BYTES;   // [Xhi; Xlo]: 2*MPAD rows of 128 B
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            const uint64_t ad = sdesc_sw128(wa + kk * 32);
-            umma_bf16(d, ad, sdesc_sw128(xh + kk * 32), idesc, (g != gstart || kk > 0) ? 1u : 0u);
-            umma_bf16(d, ad, sdesc_sw128(xl + kk * 32), idesc, 1u);
-          }
+          for (int kk = 0; kk < 4; ++kk)
+            umma_bf16(d, sdesc_sw128(wa + kk * 32), sdesc_sw128(xh + kk * 32), idesc, (g != gstart || kk > 0) ? 1u : 0u);
           umma_commit(&empty[s]);
         }
         if (!ok) break;
@@ -253,71 +289,9 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
         mbar_wait_drain(drain, 0);
       }
     }
-  } else if (warp < 4) {
-    // ------------------------------------------------ activation operand (hi/lo bf16)
-    const int tid = threadIdx.x - 64;
-    pdl_wait();
-    if (p.norm) {
-      for (int m = warp - 2; m < p.M; m += 2) {
-        const float* xr = p.x + (size_t)m * p.x_ld;
-        float ss = 0.f;
-        for (int k = lane * 4; k < p.K; k += 128) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(xr + k));
-          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        if (lane == 0) inv_rms[m] = 1.0f / sqrtf(ss / (float)p.K + p.eps);
-      }
-      named_bar_sync(2, 64);
-    }
-    int it = 0;
-    for (long long g = g0; g < g1; ++g, ++it) {
-      const int s = it % S;
-      const uint32_t ph = (it / S) & 1;
-      if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, p.err)) break;
-      const int k0 = (int)(g % p.kc) * 64;
-      uint8_t* xh = stages + (size_t)s * C::STAGE_BYTES + C::W_BYTES;
-      uint8_t* xl = xh + C::X_BYTES;
-      for (int gr = tid; gr < MPAD * 8; gr += 64) {
-        const int m = gr >> 3, c = gr & 7, k = k0 + c * 8;
-        float v[8];
-        if (m < p.M && k < p.K) {
-          const float4* src = reinterpret_cast<const float4*>(p.x + (size_t)m * p.x_ld + k);
-          const float4 a = __ldcg(src), b = __ldcg(src + 1);
-          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-          v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-          if (p.norm) {
-            const float sc = inv_rms[m];
-            const uint4 graw = *reinterpret_cast<const uint4*>(p.gain + k);
-            const __nv_bfloat16* gg = reinterpret_cast<const __nv_bfloat16*>(&graw);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) v[e] = v[e] * sc * __bfloat162float(gg[e]);
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) v[e] = 0.f;
-        }
-        uint32_t hi[4], lo[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]), h1 = __float2bfloat16_rn(v[2 * e + 1]);
-          const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * e] - __bfloat162float(h0));
-          const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1));
-          hi[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-          lo[e] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
-        }
-        const int off = m * 128 + ((c ^ (m & 7)) << 4);
-        *reinterpret_cast<uint4*>(xh + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(xl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&xfull[s]);
-    }
   } else {
     // ------------------------------------------------ epilogue (TMEM -> registers -> global)
-    const int e = warp & 3;   // TMEM lane quarter this warp may access
+    const int e = warp & 3;   // TMEM lane quarter this warp may access (warps 2-5 -> 2, 3, 0, 1)
     const int r = e * 32 + lane;
     pdl_wait();
     int seg = 0;
@@ -329,10 +303,15 @@ __global__ void __launch_bounds__(256, 2) gemm_kernel(const __grid_constant__ Ge
       if (!mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err)) break;
       tc_fence_after();
       float acc[MPAD];
+      {
+        float hl[2 * MPAD];
 #pragma unroll
-      for (int c = 0; c < MPAD; c += 16)
-        tmem_ld16(tmem + ((uint32_t)(e * 32) << 16) + buf * MPAD + c, acc + c);
-      tmem_wait_ld();
+        for (int c = 0; c < 2 * MPAD; c += 16)
+          tmem_ld16(tmem + ((uint32_t)(e * 32) << 16) + buf * C::ACC_COLS + c, hl + c);
+        tmem_wait_ld();
+#pragma unroll
+        for (int m = 0; m < MPAD; ++m) acc[m] = hl[m] + hl[MPAD + m];
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
@@ -397,11 +376,12 @@ cudaError_t gemm_prepare() {
 
 cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl) {
   const long long T = (long long)p.n_tiles * p.kc;
-  p.P = (int)std::min<long long>(num_sms, T);
   const int mpad = gemm_mpad(p.M);
+  const int per_sm = mpad <= 16 ? SDSAT_GEMM_CTAS_PER_SM : 1;
+  p.P = (int)std::min<long long>((long long)num_sms * per_sm, T);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.P);
-  cfg.blockDim = dim3(256);
+  cfg.blockDim = dim3(192);
   cfg.dynamicSmemBytes = gemm_smem_bytes(mpad);
   cfg.stream = st;
   cudaLaunchAttribute attr[1];

@@ -24,7 +24,8 @@ enum GemmEpi : int {
 };
 
 struct GemmParams {
-  CUtensorMap tmap[3];
+  CUtensorMap tmap[3];      // weights
+  CUtensorMap tmap_x[2];    // activation operand: bf16 hi and lo [rows][K], box {64, MPAD}
   int map_mode;
   int N;              // output features (MAP_GATEUP: F)
   int K;
@@ -33,16 +34,12 @@ struct GemmParams {
   int kc;             // K chunks of 64
   int P;              // CTAs
   int M;              // activation rows (<= MPAD)
-  // X source: fp32 [M][x_ld]; norm != 0 -> X = x * inv_rms(row) * gain
-  const float* x;
-  int x_ld;
-  int norm;
-  const __nv_bfloat16* gain;
-  float eps;
   // epilogue
   int epi;
   float* out;
   int out_ld;
+  __nv_bfloat16* out_hi;    // EPI_SWIGLU: the down projection's operand, hi and lo parts
+  __nv_bfloat16* out_lo;
   // EPI_QKV
   __nv_bfloat16* k_layer;   // KV cache of this layer: [B][H][cap][hd]
   __nv_bfloat16* v_layer;
@@ -64,27 +61,37 @@ cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl);
 
 // ---- attention -------------------------------------------------------------
 constexpr int ATT_CHUNK = 128;
+constexpr int ATT_MAX_CHUNKS = 256;   // contexts up to 32768 slots (the merge keeps q x chunks stats in smem)
 #define SDSAT_ATT_MAXQ 16
 struct AttnParams {
+  CUtensorMap kmap;     // the K cache as a 2-D tensor [rows][hd] bf16, boxes of 64 dims x ATT_CHUNK rows
+  CUtensorMap vmap;     // the V cache, same geometry
+  int row0;             // first row of this layer: cache row of (s, h, slot) = row0 + (s*H + h)*cap + slot
   const float* Q;       // [rows][q_ld] (row = sl*q + j), head h at column h*hd
   int q_ld;
-  const __nv_bfloat16* k;   // [B][H][cap][hd] (this layer)
-  const __nv_bfloat16* v;
   const int* len;       // [B]
   int seq0, nb, q, H, hd, cap;
-  float* out;           // [rows][out_ld]
+  float* out;           // [rows][out_ld] fp32
   int out_ld;
+  __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
+  __nv_bfloat16* out_lo;
   float* part_o;        // [rows][H][nch_max][hd]
   float* part_ml;       // [rows][H][nch_max][2]
   int nch_max;
   int* counters;        // [nb][H]
   uint32_t* err;
 };
+cudaError_t attention_prepare();   // set smem attributes (idempotent)
 cudaError_t launch_attention(const AttnParams& p, cudaStream_t st, bool pdl);
 
 // ---- embedding, acceptance, block building ------------------------------------
-cudaError_t launch_embed(const int* tokens, const __nv_bfloat16* E, int V, int d, int M, float* h,
-                         uint32_t* err, cudaStream_t st, bool pdl);
+// x = h * rsqrt(mean h^2 + eps) * g, stored as bf16 hi + lo (tokens != null: h = E[tokens] first)
+cudaError_t launch_rmsnorm(const int* tokens, const __nv_bfloat16* E, int V, float* h, int d, int M,
+                           const __nv_bfloat16* gain, float eps, __nv_bfloat16* xhi, __nv_bfloat16* xlo,
+                           uint32_t* err, cudaStream_t st, bool pdl);
+// fp32 [M][K] -> bf16 hi + lo
+cudaError_t launch_split(const float* x, int M, int K, __nv_bfloat16* xhi, __nv_bfloat16* xlo, cudaStream_t st,
+                         bool pdl);
 
 struct AcceptParams {
   const float* logits;      // [nb*q][V]

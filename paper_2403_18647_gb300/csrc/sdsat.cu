@@ -16,7 +16,7 @@
 #include <new>
 #include <vector>
 
-#include "../../include/sdsat.h"
+#include "sdsat.h"
 #include "internal.h"
 
 using namespace sdsat;
@@ -50,6 +50,32 @@ bool make_wmap(CUtensorMap* map, const void* ptr, int rows, int cols) {
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// bf16 [rows][cols] activation operand, boxes of `box_rows` rows x 64 columns, 128-byte swizzle
+bool make_xmap(CUtensorMap* map, const void* ptr, int rows, int cols, int box_rows) {
+  if (!get_encode()) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// bf16 KV cache viewed as [rows][hd], boxes of 64 dims x ATT_CHUNK rows, 128-byte swizzle
+bool make_kvmap(CUtensorMap* map, const void* ptr, long long rows, int hd) {
+  if (!get_encode()) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)hd, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)ATT_CHUNK};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int mpad_index(int M) { return M <= 16 ? 0 : (M <= 32 ? 1 : 2); }
+
 bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct LayerMaps {
@@ -58,14 +84,18 @@ struct LayerMaps {
 
 // kernel classes for the profiling hook
 enum KClass : int {
-  K_EMBED = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
+  K_RMSNORM = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
   K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_COUNT
 };
-const char* const KCLASS_NAME[K_COUNT] = {"embed", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
+const char* const KCLASS_NAME[K_COUNT] = {"rmsnorm", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
                                           "gemm_lm_head", "accept", "build_block", "kv_commit", "prefill_commit",
                                           "gemm_op", "attention_op"};
 
 constexpr int MAX_GEMM_TILES = 1 << 16;
+constexpr int OP_MAX_K = 32768;   // K limit of sdsat_op_gemm (its operand scratch is sized at create)
+
+// the GEMM activation operands (bf16 hi + lo), one pair per producer
+enum XSrc : int { X_NORM = 0, X_ATTN = 1, X_FFN = 2, X_COUNT = 3 };
 
 }  // namespace
 
@@ -95,6 +125,11 @@ struct sdsat_ctx {
   int* acc_counters = nullptr;
   int* adaptive = nullptr;
   uint32_t* err = nullptr;
+  __nv_bfloat16* x_hi[X_COUNT] = {};
+  __nv_bfloat16* x_lo[X_COUNT] = {};
+  CUtensorMap xmap[X_COUNT][3][2];     // [source][MPAD 16/32/64][hi/lo]
+  __nv_bfloat16* xop_hi = nullptr;     // operand scratch of sdsat_op_gemm
+  __nv_bfloat16* xop_lo = nullptr;
   std::vector<void*> allocs;
   // profiling hook
   bool prof = false;
@@ -110,6 +145,7 @@ struct sdsat_kv {
   __nv_bfloat16* v = nullptr;
   int* len = nullptr;
   long long* emitted = nullptr;
+  CUtensorMap kmap, vmap;   // the caches as 2-D tensors for the attention kernel
 };
 
 namespace {
@@ -153,14 +189,17 @@ sdsat_status check_cfg(const sdsat_config& c) {
   return SDSAT_OK;
 }
 
-GemmParams gemm_base(sdsat_ctx* c, int M) {
+GemmParams gemm_base(sdsat_ctx* c, int M, int xsrc) {
   GemmParams g;
   std::memset(&g, 0, sizeof(g));
   g.M = M;
   g.partials = c->partials;
   g.counters = c->gemm_counters;
   g.err = c->err;
-  g.eps = c->cfg.rms_eps;
+  if (xsrc >= 0) {
+    g.tmap_x[0] = c->xmap[xsrc][mpad_index(M)][0];
+    g.tmap_x[1] = c->xmap[xsrc][mpad_index(M)][1];
+  }
   return g;
 }
 
@@ -177,19 +216,22 @@ void set_plain(GemmParams& g, const CUtensorMap& m, int N, int K) {
 sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const int32_t* tokens,
                      const int32_t* positions, float* logits) {
   const sdsat_config& cf = c->cfg;
-  const int M = nb * q, d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd;
+  const int M = nb * q, d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd, L = cf.n_layers;
   cudaStream_t st = c->stream;
   const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
-  if (timed(c, K_EMBED, [&] {
-        return launch_embed(tokens, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, d, M, c->h, c->err,
-                            st, c->pdl);
-      }) != cudaSuccess)
-    return SDSAT_ECUDA;
-  for (int l = 0; l < cf.n_layers; ++l) {
-    const sdsat_layer_weights& W = c->layers[l];
+  auto norm = [&](const int32_t* toks, const void* gain) {
+    return timed(c, K_RMSNORM, [&] {
+      return launch_rmsnorm(toks, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, c->h, d, M,
+                            static_cast<const __nv_bfloat16*>(gain), cf.rms_eps, c->x_hi[X_NORM], c->x_lo[X_NORM],
+                            c->err, st, c->pdl);
+    });
+  };
+  // embedding gather fused with the first layer's attention RMSNorm
+  if (norm(tokens, c->layers[0].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
+  for (int l = 0; l < L; ++l) {
     const LayerMaps& mp = c->maps[l];
-    // QKV projection with the fused RMSNorm, RoPE and KV append
-    GemmParams g = gemm_base(c, M);
+    // QKV projection with RoPE and the KV append fused into its epilogue
+    GemmParams g = gemm_base(c, M, X_NORM);
     g.tmap[0] = mp.q;
     g.tmap[1] = mp.k;
     g.tmap[2] = mp.v;
@@ -199,10 +241,6 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.rows_per_map = R;
     g.n_tiles = 3 * R / 128;
     g.kc = (d + 63) / 64;
-    g.x = c->h;
-    g.x_ld = d;
-    g.norm = 1;
-    g.gain = static_cast<const __nv_bfloat16*>(W.attn_norm);
     g.epi = EPI_QKV;
     g.out = c->qbuf;
     g.out_ld = R;
@@ -218,13 +256,14 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.rope = c->rope;
     g.rope_len = cf.max_position;
     if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    // block-causal attention
+    // block-causal attention; its merge emits the O projection's operand
     AttnParams a;
     std::memset(&a, 0, sizeof(a));
+    a.kmap = kv->kmap;
+    a.vmap = kv->vmap;
+    a.row0 = l * kv->batch * H * kv->cap;
     a.Q = c->qbuf;
     a.q_ld = R;
-    a.k = kv->k + l * layer_elems;
-    a.v = kv->v + l * layer_elems;
     a.len = kv->len;
     a.seq0 = seq0;
     a.nb = nb;
@@ -234,6 +273,8 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.cap = kv->cap;
     a.out = c->attn;
     a.out_ld = R;
+    a.out_hi = c->x_hi[X_ATTN];
+    a.out_lo = c->x_lo[X_ATTN];
     a.part_o = c->att_part_o;
     a.part_ml = c->att_part_ml;
     a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
@@ -241,16 +282,15 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.err = c->err;
     if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // O projection + residual
-    g = gemm_base(c, M);
+    g = gemm_base(c, M, X_ATTN);
     set_plain(g, mp.o, d, R);
-    g.x = c->attn;
-    g.x_ld = R;
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
     if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    // gate/up with the fused RMSNorm and SiLU(gate) * up
-    g = gemm_base(c, M);
+    if (norm(nullptr, c->layers[l].ffn_norm) != cudaSuccess) return SDSAT_ECUDA;
+    // gate/up with SiLU(gate) * up fused; emits the down projection's operand
+    g = gemm_base(c, M, X_NORM);
     g.tmap[0] = mp.gate;
     g.tmap[1] = mp.up;
     g.map_mode = MAP_GATEUP;
@@ -258,35 +298,36 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.K = d;
     g.n_tiles = (F + 63) / 64;
     g.kc = (d + 63) / 64;
-    g.x = c->h;
-    g.x_ld = d;
-    g.norm = 1;
-    g.gain = static_cast<const __nv_bfloat16*>(W.ffn_norm);
     g.epi = EPI_SWIGLU;
     g.out = c->act;
     g.out_ld = F;
-    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    g.out_hi = c->x_hi[X_FFN];
+    g.out_lo = c->x_lo[X_FFN];
+    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
+      return SDSAT_ECUDA;
     // down projection + residual
-    g = gemm_base(c, M);
+    g = gemm_base(c, M, X_FFN);
     set_plain(g, mp.down, d, F);
-    g.x = c->act;
-    g.x_ld = F;
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
-    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
+      return SDSAT_ECUDA;
+    // the next layer's attention RMSNorm, or the final RMSNorm before the LM head
+    if (l + 1 < L) {
+      if (norm(nullptr, c->layers[l + 1].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
+    } else if (logits) {
+      if (norm(nullptr, c->w.final_norm) != cudaSuccess) return SDSAT_ECUDA;
+    }
   }
   if (logits) {
-    GemmParams g = gemm_base(c, M);
+    GemmParams g = gemm_base(c, M, X_NORM);
     set_plain(g, c->head_map, cf.vocab, d);
-    g.x = c->h;
-    g.x_ld = d;
-    g.norm = 1;
-    g.gain = static_cast<const __nv_bfloat16*>(c->w.final_norm);
     g.epi = EPI_STORE;
     g.out = logits;
     g.out_ld = cf.vocab;
-    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
+      return SDSAT_ECUDA;
   }
   return SDSAT_OK;
 }
@@ -367,7 +408,7 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
   }
   if (cudaGetDevice(&c->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess ||
-      gemm_prepare() != cudaSuccess) {
+      gemm_prepare() != cudaSuccess || attention_prepare() != cudaSuccess) {
     delete c;
     return SDSAT_ECUDA;
   }
@@ -414,13 +455,21 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
   c->att_nch = (cfg->max_position + ATT_CHUNK - 1) / ATT_CHUNK;
   bool ok = dalloc(c, &c->rope, rope.size()) && dalloc(c, &c->h, (size_t)rows * d) &&
             dalloc(c, &c->qbuf, (size_t)rows * R) && dalloc(c, &c->attn, (size_t)rows * R) &&
-            dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 64 * 128) &&
+            dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 2 * 64 * 128) &&
             dalloc(c, &c->gemm_counters, MAX_GEMM_TILES) &&
             dalloc(c, &c->att_part_o, (size_t)rows * cfg->n_heads * c->att_nch * cfg->head_dim) &&
             dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * c->att_nch * 2) &&
             dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
-            dalloc(c, &c->err, 1);
+            dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)rows * OP_MAX_K) &&
+            dalloc(c, &c->xop_lo, (size_t)rows * OP_MAX_K);
+  const int xcols[X_COUNT] = {d, R, F};
+  for (int xs = 0; ok && xs < X_COUNT; ++xs) {
+    ok = dalloc(c, &c->x_hi[xs], (size_t)rows * xcols[xs]) && dalloc(c, &c->x_lo[xs], (size_t)rows * xcols[xs]);
+    for (int mi = 0; ok && mi < 3; ++mi)
+      ok = make_xmap(&c->xmap[xs][mi][0], c->x_hi[xs], rows, xcols[xs], 16 << mi) &&
+           make_xmap(&c->xmap[xs][mi][1], c->x_lo[xs], rows, xcols[xs], 16 << mi);
+  }
   if (!ok) {
     sdsat_destroy(c);
     return SDSAT_ENOMEM;
@@ -447,7 +496,7 @@ sdsat_status sdsat_set_stream(sdsat_ctx* c, void* stream) {
 sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** out) {
   if (!c || !out || batch < 1 || max_len < 1) return SDSAT_EINVAL;
   *out = nullptr;
-  if (max_len > c->cfg.max_position) return SDSAT_ECAPACITY;
+  if (max_len > c->cfg.max_position || max_len > ATT_CHUNK * ATT_MAX_CHUNKS) return SDSAT_ECAPACITY;
   sdsat_kv* kv = new (std::nothrow) sdsat_kv();
   if (!kv) return SDSAT_ENOMEM;
   kv->ctx = c;
@@ -475,6 +524,16 @@ sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** ou
     return SDSAT_ECUDA;
   }
   kv->emitted = static_cast<long long*>(em);
+  const long long rows = (long long)c->cfg.n_layers * batch * c->cfg.n_heads * max_len;
+  if (rows > 0x7FFFFFFFll || !make_kvmap(&kv->kmap, k, rows, c->cfg.head_dim) ||
+      !make_kvmap(&kv->vmap, v, rows, c->cfg.head_dim)) {
+    cudaFree(k);
+    cudaFree(v);
+    cudaFree(len);
+    cudaFree(em);
+    delete kv;
+    return SDSAT_EUNSUPPORTED;
+  }
   kv->k = static_cast<__nv_bfloat16*>(k);
   kv->v = static_cast<__nv_bfloat16*>(v);
   kv->len = static_cast<int*>(len);
@@ -669,14 +728,15 @@ sdsat_status sdsat_get_error(sdsat_ctx* c, uint32_t* flags) {
 
 sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev) {
   if (!c || !x_dev || !y_dev || !aligned16(w_dev) || !aligned16(x_dev)) return SDSAT_EINVAL;
-  if (M < 1 || M > SDSAT_MAX_ROWS || K < 8 || K % 8 || N < 1 || (N + 127) / 128 > MAX_GEMM_TILES)
+  if (M < 1 || M > SDSAT_MAX_ROWS || K < 8 || K % 8 || K > OP_MAX_K || N < 1 || (N + 127) / 128 > MAX_GEMM_TILES)
     return SDSAT_EINVAL;
-  GemmParams g = gemm_base(c, M);
+  GemmParams g = gemm_base(c, M, -1);
   CUtensorMap m;
-  if (!make_wmap(&m, w_dev, N, K)) return SDSAT_ECUDA;
+  if (!make_wmap(&m, w_dev, N, K) || !make_xmap(&g.tmap_x[0], c->xop_hi, SDSAT_MAX_ROWS, K, 16 << mpad_index(M)) ||
+      !make_xmap(&g.tmap_x[1], c->xop_lo, SDSAT_MAX_ROWS, K, 16 << mpad_index(M)))
+    return SDSAT_ECUDA;
   set_plain(g, m, N, K);
-  g.x = x_dev;
-  g.x_ld = K;
+  if (launch_split(x_dev, M, K, c->xop_hi, c->xop_lo, c->stream, c->pdl) != cudaSuccess) return SDSAT_ECUDA;
   g.epi = EPI_STORE;
   g.out = y_dev;
   g.out_ld = N;
@@ -687,7 +747,8 @@ sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const
 sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_dev, const void* v_dev,
                                 const int32_t* len_dev, int b, int q, int H, int hd, int cap, float* out_dev) {
   if (!c || !q_dev || !k_dev || !v_dev || !len_dev || !out_dev) return SDSAT_EINVAL;
-  if (b < 1 || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS || (hd != 64 && hd != 128) || H < 1 || cap < 1)
+  if (b < 1 || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS || (hd != 64 && hd != 128) || H < 1 || cap < 1 ||
+      cap > ATT_CHUNK * ATT_MAX_CHUNKS)
     return SDSAT_EINVAL;
   // the split-KV workspace was sized at create for SDSAT_MAX_ROWS rows of the model's heads
   const size_t nch = (size_t)(cap + ATT_CHUNK - 1) / ATT_CHUNK;
@@ -697,10 +758,12 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
     return SDSAT_EINVAL;
   AttnParams a;
   std::memset(&a, 0, sizeof(a));
+  if (!aligned16(k_dev) || !aligned16(v_dev) || (long long)b * H * cap > 0x7FFFFFFFll) return SDSAT_EINVAL;
+  if (!make_kvmap(&a.kmap, k_dev, (long long)b * H * cap, hd) || !make_kvmap(&a.vmap, v_dev, (long long)b * H * cap, hd))
+    return SDSAT_ECUDA;
+  a.row0 = 0;
   a.Q = q_dev;
   a.q_ld = H * hd;
-  a.k = static_cast<const __nv_bfloat16*>(k_dev);
-  a.v = static_cast<const __nv_bfloat16*>(v_dev);
   a.len = len_dev;
   a.seq0 = 0;
   a.nb = b;
@@ -710,6 +773,9 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   a.cap = cap;
   a.out = out_dev;
   a.out_ld = H * hd;
+  if ((size_t)b * q * H * hd > (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * c->cfg.head_dim) return SDSAT_EINVAL;
+  a.out_hi = c->x_hi[X_ATTN];
+  a.out_lo = c->x_lo[X_ATTN];
   a.part_o = c->att_part_o;
   a.part_ml = c->att_part_ml;
   a.nch_max = (cap + ATT_CHUNK - 1) / ATT_CHUNK;
