@@ -325,7 +325,7 @@ def run_ours(args, wl, rank, world):
     # --- profiled pass (per-kernel CUDA events; launches serialised) for the roofline
     r.reset()
     n_prof = min(args.steps, steps_per_gen)
-    launches_per_step = 4 + 7 * shape.n_layers   # build, norm, 7 per layer, head, accept
+    launches_per_step = 4 + 5 * shape.n_layers   # build, embed+norm, 5 per layer, head, accept
     r.ctx.profile_begin(n_prof * (launches_per_step + 2) + 16)
     r.run_steps(n_prof, steps_per_gen, None)
     kstats = r.ctx.profile_end()

@@ -55,7 +55,7 @@ struct GemmCfg {
   static constexpr int ACC_COLS = 2 * MPAD;     // hi and lo products side by side
   static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
   static constexpr int NBAR = 2 * STAGES + 5;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + NBAR * 8 + 32;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 64 * 4 + NBAR * 8 + 32;
 };
 
 __device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
@@ -87,8 +87,42 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 
 template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
-                                               float* staging) {
+                                               float* staging, const float* sinv) {
   const int M = p.M;
+  if (p.ssq_in) {
+#pragma unroll
+    for (int m = 0; m < MPAD; ++m) acc[m] *= sinv[m];
+  }
+  if (p.epi == EPI_RESID && p.gain_next) {
+    // residual update, the next RMSNorm's operand h * g and this tile's sums of h^2
+    const int n = 128 * tile + r;
+    const bool valid = n < p.N;
+    const float gn = valid ? __bfloat162float(p.gain_next[n]) : 0.f;
+    const int e = r >> 5, lane = r & 31;
+#pragma unroll
+    for (int m = 0; m < MPAD; ++m) {
+      if (m < M) {
+        float hn = 0.f;
+        if (valid) {
+          const size_t o = (size_t)m * p.out_ld + n;
+          hn = __ldcg(p.out + o) + acc[m];
+          p.out[o] = hn;
+          const float x = hn * gn;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+          p.xn_hi[o] = hi;
+          p.xn_lo[o] = __float2bfloat16_rn(x - __bfloat162float(hi));
+        }
+        float sq = hn * hn;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+        if (lane == 0) staging[e * 64 + m] = sq;
+      }
+    }
+    named_bar_sync(1, 128);
+    if (r < M) p.ssq_out[r * p.ssq_ld + tile] = staging[r] + staging[64 + r] + staging[128 + r] + staging[192 + r];
+    named_bar_sync(1, 128);
+    return;
+  }
   if (p.epi == EPI_STORE || p.epi == EPI_RESID) {
     const int n = 128 * tile + r;
     if (n < p.N) {
@@ -167,7 +201,8 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;
   float* staging = reinterpret_cast<float*>(smem + (size_t)S * C::STAGE_BYTES);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(staging + C::STAGING);
+  float* sinv = staging + C::STAGING;   // [64] RMSNorm row factors of the operand
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sinv + 64);
   uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
   uint64_t* empty = bars + S;        // stage consumed by the tensor core
   uint64_t* acc_full = bars + 2 * S; // [2] accumulator ready
@@ -294,6 +329,17 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
     const int e = warp & 3;   // TMEM lane quarter this warp may access (warps 2-5 -> 2, 3, 0, 1)
     const int r = e * 32 + lane;
     pdl_wait();
+    if (p.ssq_in) {   // RMSNorm factor of each operand row, summed in a fixed order
+      const int n = p.M * p.ssq_n;            // <= MPAD * 64 <= the staging area
+      for (int i = r; i < n; i += 128) staging[i] = __ldcg(p.ssq_in + (i / p.ssq_n) * p.ssq_ld + i % p.ssq_n);
+      named_bar_sync(1, 128);
+      if (r < p.M) {
+        float ssum = 0.f;
+        for (int t = 0; t < p.ssq_n; ++t) ssum += staging[r * p.ssq_n + t];
+        sinv[r] = 1.0f / sqrtf(ssum / (float)p.norm_dim + p.norm_eps);
+      }
+      named_bar_sync(1, 128);
+    }
     int seg = 0;
     long long g = g0;
     while (g < g1) {
@@ -345,7 +391,7 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
         }
         if (r == 0) p.counters[tile] = 0;
       }
-      epilogue_final<MPAD>(p, tile, r, acc, staging);
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv);
     }
   }
 

@@ -40,6 +40,19 @@ struct GemmParams {
   int out_ld;
   __nv_bfloat16* out_hi;    // EPI_SWIGLU: the down projection's operand, hi and lo parts
   __nv_bfloat16* out_lo;
+  // RMSNorm folded into the GEMMs.  RMSNorm scales each row by one scalar, so the
+  // operand can be stored un-normalised (h * gain) and the consuming GEMM multiplies
+  // its result row m by rsqrt(sum_t ssq_in[m][t] / norm_dim + norm_eps).
+  const float* ssq_in;      // [M][ssq_ld] partial sums of h^2, or null (operand already normalised)
+  int ssq_n, ssq_ld;
+  int norm_dim;
+  float norm_eps;
+  // EPI_RESID producer side: with gain_next set, also emit h * gain_next as the next
+  // GEMM's bf16 hi + lo operand [M][N] and this tile's sums of h^2 into ssq_out[m][tile].
+  const __nv_bfloat16* gain_next;
+  __nv_bfloat16* xn_hi;
+  __nv_bfloat16* xn_lo;
+  float* ssq_out;
   // EPI_QKV
   __nv_bfloat16* k_layer;   // KV cache of this layer: [B][H][cap][hd]
   __nv_bfloat16* v_layer;

@@ -117,6 +117,8 @@ struct sdsat_ctx {
   float* act = nullptr;
   float* partials = nullptr;
   int* gemm_counters = nullptr;
+  float* ssq = nullptr;        // [SDSAT_MAX_ROWS][ssq_ld] per-tile sums of h^2 (RMSNorm folded into the GEMMs)
+  int ssq_ld = 0;
   float* att_part_o = nullptr;
   float* att_part_ml = nullptr;
   int att_nch = 0;
@@ -181,6 +183,7 @@ sdsat_status check_cfg(const sdsat_config& c) {
       !(c.rope_theta > 0.f))
     return SDSAT_EINVAL;
   if (c.d_model % 8 || c.ffn_dim % 8) return SDSAT_EINVAL;
+  if (c.d_model > 64 * 128) return SDSAT_EUNSUPPORTED;   // the folded RMSNorm keeps <= 64 tile sums per row
   if (c.n_kv_heads != c.n_heads) return SDSAT_EUNSUPPORTED;
   if (c.head_dim != 64 && c.head_dim != 128) return SDSAT_EUNSUPPORTED;
   if ((c.n_heads * c.head_dim) % 128) return SDSAT_EUNSUPPORTED;
@@ -226,7 +229,24 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
                             c->err, st, c->pdl);
     });
   };
-  // embedding gather fused with the first layer's attention RMSNorm
+  // The residual-producing GEMMs (O, down) also emit the next RMSNorm's operand h * g
+  // and per-tile sums of h^2; the consuming GEMM (gate/up, the next QKV, the LM head)
+  // scales its result rows by the RMSNorm factor.  Only the first norm is a kernel,
+  // fused with the embedding gather.
+  auto fold_in = [&](GemmParams& g) {
+    g.ssq_in = c->ssq;
+    g.ssq_n = c->ssq_ld;
+    g.ssq_ld = c->ssq_ld;
+    g.norm_dim = d;
+    g.norm_eps = cf.rms_eps;
+  };
+  auto fold_out = [&](GemmParams& g, const void* gain) {
+    g.gain_next = static_cast<const __nv_bfloat16*>(gain);
+    g.xn_hi = c->x_hi[X_NORM];
+    g.xn_lo = c->x_lo[X_NORM];
+    g.ssq_out = c->ssq;
+    g.ssq_ld = c->ssq_ld;
+  };
   if (norm(tokens, c->layers[0].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
   for (int l = 0; l < L; ++l) {
     const LayerMaps& mp = c->maps[l];
@@ -255,6 +275,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.positions = positions;
     g.rope = c->rope;
     g.rope_len = cf.max_position;
+    if (l > 0) fold_in(g);
     if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
     // block-causal attention; its merge emits the O projection's operand
     AttnParams a;
@@ -287,8 +308,8 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
+    fold_out(g, c->layers[l].ffn_norm);
     if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    if (norm(nullptr, c->layers[l].ffn_norm) != cudaSuccess) return SDSAT_ECUDA;
     // gate/up with SiLU(gate) * up fused; emits the down projection's operand
     g = gemm_base(c, M, X_NORM);
     g.tmap[0] = mp.gate;
@@ -303,6 +324,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.out_ld = F;
     g.out_hi = c->x_hi[X_FFN];
     g.out_lo = c->x_lo[X_FFN];
+    fold_in(g);
     if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
       return SDSAT_ECUDA;
     // down projection + residual
@@ -311,18 +333,15 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.epi = EPI_RESID;
     g.out = c->h;
     g.out_ld = d;
+    // the next layer's attention RMSNorm, or the final RMSNorm before the LM head
+    fold_out(g, l + 1 < L ? c->layers[l + 1].attn_norm : c->w.final_norm);
     if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
       return SDSAT_ECUDA;
-    // the next layer's attention RMSNorm, or the final RMSNorm before the LM head
-    if (l + 1 < L) {
-      if (norm(nullptr, c->layers[l + 1].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
-    } else if (logits) {
-      if (norm(nullptr, c->w.final_norm) != cudaSuccess) return SDSAT_ECUDA;
-    }
   }
   if (logits) {
     GemmParams g = gemm_base(c, M, X_NORM);
     set_plain(g, c->head_map, cf.vocab, d);
+    fold_in(g);
     g.epi = EPI_STORE;
     g.out = logits;
     g.out_ld = cf.vocab;
@@ -453,6 +472,7 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
     }
   const int rows = SDSAT_MAX_ROWS;
   c->att_nch = (cfg->max_position + ATT_CHUNK - 1) / ATT_CHUNK;
+  c->ssq_ld = (d + 127) / 128;
   bool ok = dalloc(c, &c->rope, rope.size()) && dalloc(c, &c->h, (size_t)rows * d) &&
             dalloc(c, &c->qbuf, (size_t)rows * R) && dalloc(c, &c->attn, (size_t)rows * R) &&
             dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 2 * 64 * 128) &&
@@ -462,6 +482,7 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
             dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
             dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)rows * OP_MAX_K) &&
+            dalloc(c, &c->ssq, (size_t)rows * ((d + 127) / 128)) &&
             dalloc(c, &c->xop_lo, (size_t)rows * OP_MAX_K);
   const int xcols[X_COUNT] = {d, R, F};
   for (int xs = 0; ok && xs < X_COUNT; ++xs) {
