@@ -264,6 +264,28 @@ SDSAT_API sdsat_status sdsat_debug_workspace(sdsat_ctx* ctx, int which, int rows
 /* out[i] = the nucleus sampler's exp (see sdsat_accept_nucleus) of in[i] <= 0. */
 SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* out_dev, int n);
 
+/* y[m][n] = sum_k x[m][k] * W[n][k] like sdsat_op_gemm, for callers that cannot
+ * allocate device memory: no context, no cudaMalloc or other allocating call.
+ * This entry point has no counterpart in the paper; it exists because a caller
+ * may be capturing a CUDA graph (where allocation is not allowed), may run inside
+ * a framework that owns all device memory through its own allocator, or may have
+ * a fixed memory budget.  Its scratch -- the operand split, the split-K partial
+ * sums and the tile counters -- is one fixed array in device memory (3 MiB +
+ * 2 KiB, held by every GPU that loads the library until the process exits).
+ *   x_dev fp32 [M][K] (16-byte aligned), W bf16 [N][K] (16-byte aligned),
+ *   y_dev fp32 [M][N]; stream is a cudaStream_t (NULL = legacy default stream).
+ *   Limits: 1 <= M <= 16, 8 <= K <= 16384 with K % 8 == 0, 1 <= N <= 65536;
+ *   sizes past the limits return ECAPACITY, malformed arguments EINVAL.
+ * The first call on a device (with that device current) looks up the array's
+ * device address and prepares the kernels; make that first call before any
+ * stream capture.  Every call shares the one array: calls whose work overlaps
+ * on the GPU (different streams, or concurrent host threads) race and must be
+ * serialised by the caller.  The call clears the tile counters it uses; the
+ * other scratch contents are overwritten before they are read.  Device-side
+ * wait timeouts are not reported by this entry point.  Asynchronous on `stream`. */
+SDSAT_API sdsat_status sdsat_gemm_static(const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev,
+                                         void* stream);
+
 /* ---- measurement ------------------------------------------------------------------ */
 
 /* Per-kernel timing: between sdsat_profile_begin and sdsat_profile_end every
