@@ -249,7 +249,7 @@ SDSAT_API sdsat_status sdsat_op_gemm(sdsat_ctx* ctx, const float* x_dev, int M, 
  * out[s*q+j][h*hd+d] = sum_t softmax_t(q_j . k_t / sqrt(hd)) v_t[d] over slots
  * t < len[s] + j + 1.  q_dev fp32 [b*q][H*hd]; k_dev, v_dev bf16
  * [b][H][cap][hd]; len_dev int32 [b] (device); out_dev fp32 [b*q][H*hd].
- * hd must be 64 or 128.  Errors: EINVAL. */
+ * hd must be 64 or 128; k_dev, v_dev and out_dev 16-byte aligned.  Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, const void* k_dev, const void* v_dev,
                                 const int32_t* len_dev, int b, int q, int H, int hd, int cap,
                                 float* out_dev);
@@ -303,6 +303,25 @@ typedef struct {
 
 SDSAT_API sdsat_status sdsat_profile_begin(sdsat_ctx* ctx, int max_launches);
 SDSAT_API sdsat_status sdsat_profile_end(sdsat_ctx* ctx, sdsat_kernel_stat* out, int max_out, int* n_out);
+
+/* Device timeline trace (does not serialise launches): between sdsat_trace_begin and
+ * sdsat_trace_end, thread 0 of every CTA of the block forward's GEMM and attention kernels
+ * appends one record of SDSAT_TRACE_WORDS uint64:
+ *   [0] tag << 32 | block index, tag = kernel class << 24 | launch sequence number
+ *       (sdsat_kernel_class_name names a class);
+ *   [1] flags << 32 | SM id;
+ *   [2] %globaltimer (ns) at kernel entry, [3] after the wait for the preceding kernel,
+ *   [4], [5], [6] kernel-specific marks (0 = not reached), [7] at exit.
+ * GEMM: marks = first MMA issued, accumulator of the CTA's last tile ready, that tile
+ * reduced (or handed to another CTA); flags = 1 if this CTA reduced it | contributors << 8.
+ * Attention: marks = K tile landed, partial result written, merge weights ready (merging
+ * CTA only); flags = 1 for the merging CTA | number of chunks << 8.
+ * begin allocates room for max_records records (call it outside any graph capture); end
+ * synchronises, copies up to max_records records to host memory and frees the buffer. */
+#define SDSAT_TRACE_WORDS 8
+SDSAT_API sdsat_status sdsat_trace_begin(sdsat_ctx* ctx, int max_records);
+SDSAT_API sdsat_status sdsat_trace_end(sdsat_ctx* ctx, uint64_t* records_host, int max_records, int* n_records);
+SDSAT_API const char* sdsat_kernel_class_name(int kernel_class);
 
 #ifdef __cplusplus
 }

@@ -22,6 +22,7 @@ from . import build as _build
 MAX_Q = 16
 MAX_ROWS = 64
 MAX_ADAPTIVE = 16
+TRACE_WORDS = 8        # words per device trace record
 
 DEV_NAN_LOGITS = 0x1
 DEV_TIMEOUT = 0x2
@@ -83,6 +84,8 @@ def _lib():
             "sdsat_kv_lengths": [P, P, P, I],
             "sdsat_kv_emitted": [P, P, P, I, I],
             "sdsat_profile_begin": [P, I],
+            "sdsat_trace_begin": [P, I],
+            "sdsat_trace_end": [P, P, I, ctypes.POINTER(I)],
             "sdsat_profile_end": [P, ctypes.POINTER(KernelStat), I, ctypes.POINTER(I)],
             "sdsat_build_block": [P, P, I, P, P, P, I, I, I, P],
             "sdsat_prefill": [P, P, I, P, I],
@@ -100,6 +103,8 @@ def _lib():
         lib.sdsat_destroy.restype = None
         lib.sdsat_kv_destroy.argtypes = [P]
         lib.sdsat_kv_destroy.restype = None
+        lib.sdsat_kernel_class_name.argtypes = [ctypes.c_int]
+        lib.sdsat_kernel_class_name.restype = ctypes.c_char_p
         lib.sdsat_status_string.argtypes = [ctypes.c_int]
         lib.sdsat_status_string.restype = ctypes.c_char_p
         _LIB = lib
@@ -271,6 +276,25 @@ class Context:
         n = ctypes.c_int(0)
         _check(_lib().sdsat_profile_end(self.handle, buf, 32, ctypes.byref(n)), "sdsat_profile_end")
         return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].total_ms)) for i in range(n.value)}
+
+    def trace_begin(self, max_records: int):
+        _check(_lib().sdsat_trace_begin(self.handle, max_records), "sdsat_trace_begin")
+
+    def trace_end(self, max_records: int):
+        """Device timeline records: list of dicts with the kernel class name, launch seq, block,
+        smid, flags and the %globaltimer stamps entry / wait / marks (3) / exit."""
+        import numpy as np
+        buf = np.zeros((max_records, TRACE_WORDS), dtype=np.uint64)
+        n = ctypes.c_int(0)
+        self._bind_stream()
+        _check(_lib().sdsat_trace_end(self.handle, buf.ctypes.data, max_records, ctypes.byref(n)), "sdsat_trace_end")
+        out = []
+        for r in buf[:n.value]:
+            tag, blk = int(r[0]) >> 32, int(r[0]) & 0xFFFFFFFF
+            out.append(dict(kernel=_lib().sdsat_kernel_class_name(tag >> 24).decode(), seq=tag & 0xFFFFFF,
+                            block=blk, smid=int(r[1]) & 0xFFFFFFFF, flags=int(r[1]) >> 32, entry=int(r[2]),
+                            wait=int(r[3]), marks=(int(r[4]), int(r[5]), int(r[6])), exit=int(r[7])))
+        return out
 
     def build_block(self, kv: KV, mode: int, prev_out, prev_acc, tokens_out, b: int, q: int,
                     draft_table=None, table_stride: int = 0):

@@ -84,6 +84,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, tig = lane & 3;
   const int q = p.q;
+  const unsigned long long t_entry = p.trace.rec ? globaltimer_ns() : 0;
   pdl_trigger();
   // The committed length is final before this kernel can start: the block forward's
   // first kernel (RMSNorm) lets its dependents launch only after every earlier kernel
@@ -113,6 +114,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     if (early) issue_loads();
   }
   pdl_wait();   // q and this forward's new K/V rows come from the QKV projection
+  const unsigned long long t_wait = p.trace.rec ? globaltimer_ns() : 0;
   if (tid == 0 && !early) issue_loads();
   // q (scaled by 1/sqrt(hd)) as bf16 hi + lo; rows >= q are zero
   const float scale = rsqrtf((float)HD);
@@ -134,6 +136,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
 
   volatile int no_abort = 0;
   bool ok = mbar_wait_bounded(&bar[0], 0, &no_abort, p.err);
+  const unsigned long long t_k = p.trace.rec ? globaltimer_ns() : 0;
 
   // ---- S = Q K^T for this warp's 32 keys (4 tiles of 8), fp32 in registers
   const int kb = warp * 32;                       // first key (within the chunk) of this warp
@@ -279,59 +282,116 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   }
 
   // the last chunk CTA of this (sequence, head) merges the chunks
+  const unsigned long long t_part = p.trace.rec ? globaltimer_ns() : 0;
   __threadfence();
   __syncthreads();
   if (tid == 0) *s_last = (atomicAdd(p.counters + sl * p.H + h, 1) == nch - 1);
   __syncthreads();
-  if (!*s_last) return;
+  if (!*s_last) {
+    if (tid == 0 && p.trace.rec)
+      trace_write(p.trace, (unsigned)nch << 8, t_entry, t_wait, t_k, t_part, 0, globaltimer_ns());
+    return;
+  }
   __threadfence();
-  // chunk statistics of every row -> shared memory (the K tile is free now), then the
-  // per-row rescaling weights w[j][c] = exp(m_c - max_c m_c) and the normaliser L_j
-  float* w = reinterpret_cast<float*>(Ktile);          // [q][nch]; q*nch <= 16 * ATT_MAX_CHUNKS
-  float* lsum = w + q * nch;                            // [q][nch]; both fit the K + V tiles
-  for (int i = tid; i < q * nch; i += 128) {
-    const int j = i / nch, c = i % nch;
-    const float* ml = p.part_ml + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max + c) * 2;
-    w[i] = __ldcg(ml);
-    lsum[i] = __ldcg(ml + 1);
-  }
-  __syncthreads();
-  if (tid < q) {
-    float mx = -INFINITY;
-    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, w[tid * nch + c]);
-    float L = 0.f;
-    for (int c = 0; c < nch; ++c) {
-      const float mc = w[tid * nch + c];
-      const float wc = (mc == -INFINITY) ? 0.f : expf(mc - mx);
-      w[tid * nch + c] = wc;
-      L += wc * lsum[tid * nch + c];
-    }
-    Ms[tid] = 1.0f / L;
-  }
-  __syncthreads();
-  if (tid < HD) {
-    for (int j = 0; j < q; ++j) {
-      const float* po = p.part_o + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max) * HD + tid;
-      float O = 0.f;
-      int c = 0;
-      for (; c + 4 <= nch; c += 4) {   // four independent loads in flight
-        const float o0 = __ldcg(po + (size_t)c * HD), o1 = __ldcg(po + (size_t)(c + 1) * HD);
-        const float o2 = __ldcg(po + (size_t)(c + 2) * HD), o3 = __ldcg(po + (size_t)(c + 3) * HD);
-        O += w[j * nch + c] * o0;
-        O += w[j * nch + c + 1] * o1;
-        O += w[j * nch + c + 2] * o2;
-        O += w[j * nch + c + 3] * o3;
+  // Merge weights: warp w takes rows j = w, w + 4, ...; its lanes hold the chunks.
+  // w[j][c] = exp(m_c - max_c m_c) goes to shared memory (the K tile is free now),
+  // 1 / L_j with L_j = sum_c w[j][c] l_c to Ms[j].
+  float* wgt = reinterpret_cast<float*>(Ktile);   // [q][nch]; q * nch <= 16 * ATT_MAX_CHUNKS floats
+  constexpr int CPL = ATT_MAX_CHUNKS / 32;        // chunks per lane
+  for (int j = warp; j < q; j += 4) {
+    const float* mlr = p.part_ml + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max) * 2;
+    float mc[CPL], lc[CPL];
+#pragma unroll
+    for (int u = 0; u < CPL; ++u) {
+      const int c = lane + 32 * u;
+      mc[u] = -INFINITY;
+      lc[u] = 0.f;
+      if (c < nch) {
+        const float2 v = __ldcg(reinterpret_cast<const float2*>(mlr) + c);
+        mc[u] = v.x;
+        lc[u] = v.y;
       }
-      for (; c < nch; ++c) O += w[j * nch + c] * __ldcg(po + (size_t)c * HD);
-      const float o = O * Ms[j];
-      const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + tid;
-      p.out[idx] = o;
-      const __nv_bfloat16 hi = __float2bfloat16_rn(o);
-      p.out_hi[idx] = hi;
-      p.out_lo[idx] = __float2bfloat16_rn(o - __bfloat162float(hi));
+    }
+    float mx = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < CPL; ++u) mx = fmaxf(mx, mc[u]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float L = 0.f;
+#pragma unroll
+    for (int u = 0; u < CPL; ++u) {
+      const int c = lane + 32 * u;
+      const float wc = (mc[u] == -INFINITY) ? 0.f : expf(mc[u] - mx);
+      if (c < nch) wgt[j * nch + c] = wc;
+      L += wc * lc[u];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (lane == 0) Ms[j] = 1.0f / L;
+  }
+  __syncthreads();
+  const unsigned long long t_stats = p.trace.rec ? globaltimer_ns() : 0;
+  // O_j = (sum_c w[j][c] o_c) / L_j: thread = (row group, 4 dimensions); every row of the
+  // group advances four chunks at a time, so up to 16 float4 loads are in flight
+  {
+    constexpr int D4 = HD / 4;                 // float4 columns of a row
+    constexpr int RG = 128 / D4;               // row groups
+    constexpr int RPT = (16 + RG - 1) / RG;    // rows per thread (q <= 16)
+    const int d4 = tid % D4, jg = tid / D4;
+    float4 acc[RPT];
+#pragma unroll
+    for (int k = 0; k < RPT; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c0 = 0; c0 < nch; c0 += 4) {
+      float4 v[RPT][4];
+#pragma unroll
+      for (int k = 0; k < RPT; ++k) {
+        const int j = jg + RG * k;
+        const float4* po = reinterpret_cast<const float4*>(
+                               p.part_o + ((size_t)(sl * q + j) * p.H * p.nch_max + (size_t)h * p.nch_max) * HD) + d4;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (j < q && c0 + u < nch) v[k][u] = __ldcg(po + (size_t)(c0 + u) * D4);
+      }
+#pragma unroll
+      for (int k = 0; k < RPT; ++k) {
+        const int j = jg + RG * k;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          if (j < q && c0 + u < nch) {
+            const float wc = wgt[j * nch + c0 + u];
+            acc[k].x += wc * v[k][u].x;
+            acc[k].y += wc * v[k][u].y;
+            acc[k].z += wc * v[k][u].z;
+            acc[k].w += wc * v[k][u].w;
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < RPT; ++k) {
+      const int j = jg + RG * k;
+      if (j < q) {
+        const float inv = Ms[j];
+        const float4 o = make_float4(acc[k].x * inv, acc[k].y * inv, acc[k].z * inv, acc[k].w * inv);
+        const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + 4 * d4;
+        *reinterpret_cast<float4*>(p.out + idx) = o;
+        const __nv_bfloat16 h0 = __float2bfloat16_rn(o.x), h1 = __float2bfloat16_rn(o.y);
+        const __nv_bfloat16 h2 = __float2bfloat16_rn(o.z), h3 = __float2bfloat16_rn(o.w);
+        uint2 hi, lo;
+        hi.x = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+        hi.y = (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
+        lo.x = pack_bf16(o.x - __bfloat162float(h0), o.y - __bfloat162float(h1));
+        lo.y = pack_bf16(o.z - __bfloat162float(h2), o.w - __bfloat162float(h3));
+        *reinterpret_cast<uint2*>(p.out_hi + idx) = hi;
+        *reinterpret_cast<uint2*>(p.out_lo + idx) = lo;
+      }
     }
   }
-  if (tid == 0) p.counters[sl * p.H + h] = 0;
+  if (tid == 0) {
+    p.counters[sl * p.H + h] = 0;
+    if (p.trace.rec)
+      trace_write(p.trace, 1u | ((unsigned)nch << 8), t_entry, t_wait, t_k, t_part, t_stats, globaltimer_ns());
+  }
 }
 
 size_t attention_smem_bytes(int hd) { return hd == 64 ? AttCfg<64>::SMEM : AttCfg<128>::SMEM; }

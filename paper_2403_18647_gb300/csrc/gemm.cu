@@ -44,6 +44,18 @@ namespace sdsat {
 #ifndef SDSAT_GEMM_CTAS_PER_SM
 #define SDSAT_GEMM_CTAS_PER_SM 2
 #endif
+// Minimum resident CTAs per SM the register allocation must allow (192 threads each).
+// The M <= 16 kernel stays below 112 registers without it (-Xptxas -v), so a third CTA
+// -- the next kernel's, launched early by programmatic dependent launch -- fits beside
+// two running ones and prefetches its weights.
+#ifndef SDSAT_GEMM_MINB
+#define SDSAT_GEMM_MINB 2
+#endif
+// Epilogue rows handled per group: a group's loads are all issued before its stores.
+#ifndef SDSAT_GEMM_EPI_GROUP
+#define SDSAT_GEMM_EPI_GROUP 8
+#endif
+constexpr int EG = SDSAT_GEMM_EPI_GROUP;
 
 template <int MPAD>
 struct GemmCfg {
@@ -54,8 +66,8 @@ struct GemmCfg {
   static constexpr int STAGING = 128 * (MPAD + 1);
   static constexpr int ACC_COLS = 2 * MPAD;     // hi and lo products side by side
   static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
-  static constexpr int NBAR = 2 * STAGES + 5;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 64 * 4 + NBAR * 8 + 32;
+  static constexpr int NBAR = 2 * STAGES + 6;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + NBAR * 8 + 64;
 };
 
 __device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
@@ -63,14 +75,14 @@ __device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int 
 }
 
 // (tensor map, first row) of half h (0: tile rows 0-63, 1: rows 64-127) of tile t
-__device__ __forceinline__ void tile_half_src(const GemmParams& p, int t, int h, int& map, int& row) {
-  if (p.map_mode == MAP_GATEUP) {
+__device__ __forceinline__ void tile_half_src(int map_mode, int rows_per_map, int t, int h, int& map, int& row) {
+  if (map_mode == MAP_GATEUP) {
     map = h;
     row = 64 * t;
-  } else if (p.map_mode == MAP_QKV3) {
+  } else if (map_mode == MAP_QKV3) {
     const int g = 128 * t;
-    map = g / p.rows_per_map;
-    row = g % p.rows_per_map + 64 * h;
+    map = g / rows_per_map;
+    row = g % rows_per_map + 64 * h;
   } else {
     map = 0;
     row = 128 * t + 64 * h;
@@ -87,7 +99,8 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 
 template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
-                                               float* staging, const float* sinv) {
+                                               float* staging, const float* sinv, const int* s_slot,
+                                               const int* s_pos, const float (&pre)[EG], float pre_gn) {
   const int M = p.M;
   if (p.ssq_in) {
 #pragma unroll
@@ -97,15 +110,22 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     // residual update, the next RMSNorm's operand h * g and this tile's sums of h^2
     const int n = 128 * tile + r;
     const bool valid = n < p.N;
-    const float gn = valid ? __bfloat162float(p.gain_next[n]) : 0.f;
+    const float gn = pre_gn;
     const int e = r >> 5, lane = r & 31;
 #pragma unroll
-    for (int m = 0; m < MPAD; ++m) {
-      if (m < M) {
+    for (int m0 = 0; m0 < MPAD; m0 += EG) {
+      float hv[EG];   // a group's residual rows are loaded before anything is stored (group 0: earlier)
+#pragma unroll
+      for (int u = 0; u < EG; ++u)
+        hv[u] = m0 == 0 ? pre[u] : (m0 + u < M && valid) ? __ldcg(p.out + (size_t)(m0 + u) * p.out_ld + n) : 0.f;
+#pragma unroll
+      for (int u = 0; u < EG; ++u) {
+        const int m = m0 + u;
+        if (m >= M) break;
         float hn = 0.f;
         if (valid) {
           const size_t o = (size_t)m * p.out_ld + n;
-          hn = __ldcg(p.out + o) + acc[m];
+          hn = hv[u] + acc[m];
           p.out[o] = hn;
           const float x = hn * gn;
           const __nv_bfloat16 hi = __float2bfloat16_rn(x);
@@ -126,13 +146,20 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
   if (p.epi == EPI_STORE || p.epi == EPI_RESID) {
     const int n = 128 * tile + r;
     if (n < p.N) {
+      if (p.epi == EPI_RESID) {
 #pragma unroll
-      for (int m = 0; m < MPAD; ++m) {
-        if (m < M) {
-          float* o = p.out + (size_t)m * p.out_ld + n;
-          *o = (p.epi == EPI_RESID) ? __ldcg(o) + acc[m] : acc[m];
+        for (int m0 = 0; m0 < MPAD; m0 += EG) {
+          float hv[EG];
+#pragma unroll
+          for (int u = 0; u < EG; ++u)
+            hv[u] = m0 == 0 ? pre[u] : (m0 + u < M) ? __ldcg(p.out + (size_t)(m0 + u) * p.out_ld + n) : 0.f;
+#pragma unroll
+          for (int u = 0; u < EG; ++u) acc[m0 + u] += hv[u];
         }
       }
+#pragma unroll
+      for (int m = 0; m < MPAD; ++m)
+        if (m < M) p.out[(size_t)m * p.out_ld + n] = acc[m];
     }
     return;
   }
@@ -164,29 +191,39 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int head = f / hd, i = f % hd;
     const int partner = (i < half) ? r + half : r - half;
 #pragma unroll
-    for (int m = 0; m < MPAD; ++m) {
-      if (m >= M) break;
-      const int sl = m / p.q, j = m % p.q, s = p.seq0 + sl;
-      const int slot = __ldcg(p.len + s) + j;
-      const float x = acc[m];
-      float val = x;
-      if (which < 2) {
-        int pos = p.positions ? __ldcg(p.positions + m) : slot;
-        if (pos < 0 || pos >= p.rope_len) {
-          set_error(p.err, ERR_POSITION);
-          pos = pos < 0 ? 0 : p.rope_len - 1;
+    for (int m0 = 0; m0 < MPAD; m0 += EG) {
+      // a group's RoPE factors first, so no load waits behind a store
+      int slot[EG];
+      float2 cs[EG];
+#pragma unroll
+      for (int u = 0; u < EG; ++u) {
+        const int m = m0 + u;
+        slot[u] = 0;
+        cs[u] = make_float2(1.f, 0.f);
+        if (m < M) {
+          slot[u] = s_slot[m];
+          if (which < 2) cs[u] = p.rope[(size_t)s_pos[m] * half + (i % half)];
         }
-        const float y = staging[partner * (MPAD + 1) + m];
-        const float2 cs = p.rope[(size_t)pos * half + (i % half)];
-        val = (i < half) ? x * cs.x - y * cs.y : x * cs.x + y * cs.y;
       }
-      if (which == 0) {
-        p.out[(size_t)m * p.out_ld + f] = val;
-      } else if (slot < p.cap) {
-        __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
-        cache[(((size_t)s * p.H + head) * p.cap + slot) * hd + i] = __float2bfloat16_rn(val);
-      } else if (i == 0 && which == 1) {
-        set_error(p.err, ERR_CAPACITY);
+#pragma unroll
+      for (int u = 0; u < EG; ++u) {
+        const int m = m0 + u;
+        if (m >= M) break;
+        const int s = p.seq0 + m / p.q;
+        const float x = acc[m];
+        float val = x;
+        if (which < 2) {
+          const float y = staging[partner * (MPAD + 1) + m];
+          val = (i < half) ? x * cs[u].x - y * cs[u].y : x * cs[u].x + y * cs[u].y;
+        }
+        if (which == 0) {
+          p.out[(size_t)m * p.out_ld + f] = val;
+        } else if (slot[u] < p.cap) {
+          __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
+          cache[(((size_t)s * p.H + head) * p.cap + slot[u]) * hd + i] = __float2bfloat16_rn(val);
+        } else if (i == 0 && which == 1) {
+          set_error(p.err, ERR_CAPACITY);
+        }
       }
     }
   }
@@ -194,7 +231,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
 }
 
 template <int MPAD>
-__global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ GemmParams p) {
+__global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid_constant__ GemmParams p) {
   using C = GemmCfg<MPAD>;
   constexpr int S = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -202,19 +239,26 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
   uint8_t* stages = smem;
   float* staging = reinterpret_cast<float*>(smem + (size_t)S * C::STAGE_BYTES);
   float* sinv = staging + C::STAGING;   // [64] RMSNorm row factors of the operand
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sinv + 64);
+  int* s_slot = reinterpret_cast<int*>(sinv + 64);   // [64] EPI_QKV: cache slot of each row
+  int* s_pos = s_slot + 64;                          // [64] EPI_QKV: RoPE position of each row
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_pos + 64);
   uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
   uint64_t* empty = bars + S;        // stage consumed by the tensor core
   uint64_t* acc_full = bars + 2 * S; // [2] accumulator ready
   uint64_t* acc_empty = acc_full + 2;// [2] accumulator drained
   uint64_t* drain = acc_empty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* red_bar = drain + 1;     // partials of the tile being reduced landed (bulk copies)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(red_bar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* s_last = reinterpret_cast<int*>(tmem_slot + 2);
+  // trace marks: first MMA issued, last accumulator ready, last tile reduced; [3] = flags
+  unsigned long long* s_mark = reinterpret_cast<unsigned long long*>(tmem_slot + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int cta = blockIdx.x;
   const long long T = (long long)p.n_tiles * p.kc;
+  const unsigned long long t_entry = p.trace.rec ? globaltimer_ns() : 0;
+  unsigned long long t_wait = 0;
   const long long g0 = (long long)cta * T / p.P, g1 = (long long)(cta + 1) * T / p.P;
 
   if (threadIdx.x == 0) {
@@ -227,7 +271,9 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
       mbar_init(&acc_empty[b], 4);
     }
     mbar_init(drain, 1);
+    mbar_init(red_bar, 1);
     *abort_flag = 0;
+    s_mark[0] = s_mark[1] = s_mark[2] = s_mark[3] = 0;
     fence_mbar_init();
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -256,7 +302,7 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           int map, row;
-          tile_half_src(p, tile, h, map, row);
+          tile_half_src(p.map_mode, p.rows_per_map, tile, h, map, row);
           tma_load_2d(dst + h * 8192, &p.tmap[map], &full[it % S], kc * 64, row, pol_w);
         }
       };
@@ -272,6 +318,7 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
         load_w(it);
       }
       pdl_wait();   // the activations are the previous kernel's output
+      if (p.trace.rec) t_wait = globaltimer_ns();
       for (int it = 0; it < npre; ++it) load_x(it);
       int it = npre;
       for (; it < n; ++it) {
@@ -308,6 +355,7 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
             break;
           }
           tc_fence_after();
+          if (it == 0 && p.trace.rec) s_mark[0] = globaltimer_ns();
           const uint32_t wa = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
           const uint32_t xh = wa + C::W_BYTES;   // [Xhi; Xlo]: 2*MPAD rows of 128 B
 #pragma unroll
@@ -340,14 +388,40 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
       }
       named_bar_sync(1, 128);
     }
+    if (p.epi == EPI_QKV) {   // cache slot and RoPE position of every row (fixed during the forward)
+      if (r < p.M) {
+        const int slot = __ldcg(p.len + p.seq0 + r / p.q) + r % p.q;
+        int pos = p.positions ? __ldcg(p.positions + r) : slot;
+        if (pos < 0 || pos >= p.rope_len) {
+          set_error(p.err, ERR_POSITION);
+          pos = pos < 0 ? 0 : p.rope_len - 1;
+        }
+        s_slot[r] = slot;
+        s_pos[r] = pos;
+      }
+      named_bar_sync(1, 128);
+    }
     int seg = 0;
     long long g = g0;
     while (g < g1) {
       const int tile = (int)(g / p.kc);
       g = std::min(g1, (long long)(tile + 1) * p.kc);
       const int buf = seg & 1;
+      // the residual rows (first group) and gain this tile's epilogue needs, loaded while
+      // the tensor cores work
+      float pre[EG];
+      float pre_gn = 0.f;
+      {
+        const int n = 128 * tile + r;
+        const bool resid = p.epi == EPI_RESID && n < p.N;
+#pragma unroll
+        for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
+        if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
+      }
       if (!mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err)) break;
       tc_fence_after();
+      const bool last_seg = g >= g1;
+      if (r == 0 && last_seg && p.trace.rec) s_mark[1] = globaltimer_ns();
       float acc[MPAD];
       {
         float hl[2 * MPAD];
@@ -374,24 +448,69 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
 #pragma unroll
         for (int m = 0; m < MPAD; ++m)
           if (m < p.M) mine[m * 128 + r] = acc[m];
-        __threadfence();
+        // publish: the CTA's stores, then one release/acquire counter update (thread r = 0)
         named_bar_sync(1, 128);
-        if (r == 0) *s_last = (atomicAdd(&p.counters[tile], 1) == c_hi - c_lo);
+        if (r == 0) {
+          __threadfence();
+          *s_last = (atomicAdd(&p.counters[tile], 1) == c_hi - c_lo);
+          __threadfence();
+        }
         named_bar_sync(1, 128);
-        if (!*s_last) continue;
-        __threadfence();
+        if (r == 0 && last_seg && p.trace.rec) s_mark[3] = (unsigned long long)(*s_last) | ((c_hi - c_lo + 1) << 8);
+        if (!*s_last) {
+          if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
+          continue;
+        }
 #pragma unroll
         for (int m = 0; m < MPAD; ++m) acc[m] = 0.f;
-        for (int j = c_lo; j <= c_hi; ++j) {
-          const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
-          const float* src = p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128;
+        const uint32_t pbytes = (uint32_t)p.M * 512;   // rows m < M of a [MPAD][128] fp32 partial
+        if (last_seg) {
+          // The stage ring is idle after the CTA's last tile (every TMA load landed and every
+          // MMA that read it completed): bulk-copy the contributors' partials into it, as many
+          // per round as fit, and sum them in CTA order.
+          const int per = max(1, (int)((S * C::STAGE_BYTES) / pbytes));
+          const float* ring = reinterpret_cast<const float*>(stages);
+          uint32_t ph = 0;
+          bool ok = true;
+          for (int j0 = c_lo; j0 <= c_hi && ok; j0 += per) {
+            const int cnt = min(per, c_hi - j0 + 1);
+            named_bar_sync(1, 128);   // the previous round's shared-memory reads are done
+            if (r == 0) {
+              fence_proxy_async_global();
+              mbar_arrive_expect_tx(red_bar, (uint32_t)cnt * pbytes);
+              for (int u = 0; u < cnt; ++u) {
+                const int j = j0 + u;
+                const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
+                bulk_load_g2s(stages + (size_t)u * pbytes,
+                              p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128, pbytes, red_bar);
+              }
+            }
+            ok = mbar_wait_bounded(red_bar, ph, abort_flag, p.err);
+            ph ^= 1u;
+            if (ok) {
+              for (int u = 0; u < cnt; ++u) {
 #pragma unroll
-          for (int m = 0; m < MPAD; ++m)
-            if (m < p.M) acc[m] += __ldcg(src + m * 128 + r);
+                for (int m = 0; m < MPAD; ++m)
+                  if (m < p.M) acc[m] += ring[(size_t)u * p.M * 128 + m * 128 + r];
+              }
+            } else if (r == 0) {
+              mbar_wait_drain(red_bar, ph ^ 1u);   // copies in flight land before the CTA exits
+            }
+          }
+          if (!ok) break;
+        } else {
+          for (int j = c_lo; j <= c_hi; ++j) {
+            const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
+            const float* src = p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128;
+#pragma unroll
+            for (int m = 0; m < MPAD; ++m)
+              if (m < p.M) acc[m] += __ldcg(src + m * 128 + r);
+          }
         }
         if (r == 0) p.counters[tile] = 0;
       }
-      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv);
+      if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn);
     }
   }
 
@@ -401,6 +520,8 @@ __global__ void __launch_bounds__(192, 2) gemm_kernel(const __grid_constant__ Ge
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
+  if (threadIdx.x == 0 && p.trace.rec)
+    trace_write(p.trace, (unsigned)s_mark[3], t_entry, t_wait, s_mark[0], s_mark[1], s_mark[2], globaltimer_ns());
 }
 
 int gemm_mpad(int M) { return M <= 16 ? 16 : (M <= 32 ? 32 : 64); }
@@ -420,11 +541,15 @@ cudaError_t gemm_prepare() {
                               (int)GemmCfg<64>::SMEM);
 }
 
-cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl) {
+static int gemm_grid(const GemmParams& p, int num_sms) {
   const long long T = (long long)p.n_tiles * p.kc;
+  const int per_sm = gemm_mpad(p.M) <= 16 ? SDSAT_GEMM_CTAS_PER_SM : 1;
+  return (int)std::min<long long>((long long)num_sms * per_sm, T);
+}
+
+cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl) {
   const int mpad = gemm_mpad(p.M);
-  const int per_sm = mpad <= 16 ? SDSAT_GEMM_CTAS_PER_SM : 1;
-  p.P = (int)std::min<long long>((long long)num_sms * per_sm, T);
+  p.P = gemm_grid(p, num_sms);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.P);
   cfg.blockDim = dim3(192);

@@ -8,6 +8,38 @@
 
 namespace sdsat {
 
+// ---- opt-in device trace: thread 0 of every CTA appends one record of TRACE_WORDS words:
+// [0] tag << 32 | block, [1] flags << 32 | SM id, [2] t_entry, [3] t_after_wait,
+// [4..6] three kernel-specific marks, [7] t_exit (%globaltimer, ns; 0 = not reached)
+constexpr int TRACE_WORDS = 8;
+struct Trace {
+  unsigned long long* rec;   // [cap][TRACE_WORDS]
+  unsigned int* count;
+  unsigned int cap;
+  unsigned int tag;          // kernel class << 24 | launch sequence number
+};
+__device__ __forceinline__ unsigned int sm_id() {
+  unsigned int r;
+  asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void trace_write(const Trace& t, unsigned int flags, unsigned long long t0,
+                                            unsigned long long tw, unsigned long long m0, unsigned long long m1,
+                                            unsigned long long m2, unsigned long long t1) {
+  if (!t.rec) return;
+  const unsigned int i = atomicAdd(t.count, 1u);
+  if (i >= t.cap) return;
+  unsigned long long* r = t.rec + (size_t)i * TRACE_WORDS;
+  r[0] = ((unsigned long long)t.tag << 32) | blockIdx.x;
+  r[1] = ((unsigned long long)flags << 32) | sm_id();
+  r[2] = t0;
+  r[3] = tw;
+  r[4] = m0;
+  r[5] = m1;
+  r[6] = m2;
+  r[7] = t1;
+}
+
 // ---- skinny weight-streaming GEMM --------------------------------------------
 // Tiles of 128 output features x 64 K-elements; the 128 rows come from two
 // 64-row TMA boxes ("halves") whose source depends on the map mode.
@@ -65,6 +97,7 @@ struct GemmParams {
   float* partials;          // [P][2][MPAD][128]
   int* counters;            // [n_tiles], zero between launches
   uint32_t* err;
+  Trace trace;
 };
 
 int gemm_mpad(int M);                 // 16, 32 or 64
@@ -93,6 +126,7 @@ struct AttnParams {
   int nch_max;
   int* counters;        // [nb][H]
   uint32_t* err;
+  Trace trace;
 };
 cudaError_t attention_prepare();   // set smem attributes (idempotent)
 cudaError_t launch_attention(const AttnParams& p, cudaStream_t st, bool pdl);

@@ -20,6 +20,7 @@
 #include "internal.h"
 
 using namespace sdsat;
+static_assert(TRACE_WORDS == SDSAT_TRACE_WORDS, "trace record size");
 
 namespace {
 
@@ -133,6 +134,11 @@ struct sdsat_ctx {
   __nv_bfloat16* xop_hi = nullptr;     // operand scratch of sdsat_op_gemm
   __nv_bfloat16* xop_lo = nullptr;
   std::vector<void*> allocs;
+  // device trace (opt-in)
+  unsigned long long* trace_rec = nullptr;
+  unsigned int* trace_count = nullptr;
+  unsigned int trace_cap = 0;
+  unsigned int trace_seq = 0;
   // profiling hook
   bool prof = false;
   std::vector<cudaEvent_t> prof_events;
@@ -151,6 +157,18 @@ struct sdsat_kv {
 };
 
 namespace {
+
+// trace descriptor for the next launch of kernel class `cls` (empty when tracing is off)
+Trace next_trace(sdsat_ctx* c, int cls) {
+  Trace t{};
+  if (c->trace_rec) {
+    t.rec = c->trace_rec;
+    t.count = c->trace_count;
+    t.cap = c->trace_cap;
+    t.tag = ((unsigned)cls << 24) | (c->trace_seq++ & 0xFFFFFFu);
+  }
+  return t;
+}
 
 // Run one kernel launch, bracketed by profiling events when the hook is on.
 template <typename F>
@@ -247,10 +265,9 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.ssq_out = c->ssq;
     g.ssq_ld = c->ssq_ld;
   };
-  if (norm(tokens, c->layers[0].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
-  for (int l = 0; l < L; ++l) {
+  // QKV projection with RoPE and the KV append fused into its epilogue
+  auto make_qkv = [&](int l) {
     const LayerMaps& mp = c->maps[l];
-    // QKV projection with RoPE and the KV append fused into its epilogue
     GemmParams g = gemm_base(c, M, X_NORM);
     g.tmap[0] = mp.q;
     g.tmap[1] = mp.k;
@@ -276,7 +293,67 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     g.rope = c->rope;
     g.rope_len = cf.max_position;
     if (l > 0) fold_in(g);
-    if (timed(c, K_GEMM_QKV, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    return g;
+  };
+  // O projection + residual
+  auto make_o = [&](int l) {
+    GemmParams g = gemm_base(c, M, X_ATTN);
+    set_plain(g, c->maps[l].o, d, R);
+    g.epi = EPI_RESID;
+    g.out = c->h;
+    g.out_ld = d;
+    fold_out(g, c->layers[l].ffn_norm);
+    return g;
+  };
+  // gate/up with SiLU(gate) * up fused; emits the down projection's operand
+  auto make_gateup = [&](int l) {
+    GemmParams g = gemm_base(c, M, X_NORM);
+    g.tmap[0] = c->maps[l].gate;
+    g.tmap[1] = c->maps[l].up;
+    g.map_mode = MAP_GATEUP;
+    g.N = F;
+    g.K = d;
+    g.n_tiles = (F + 63) / 64;
+    g.kc = (d + 63) / 64;
+    g.epi = EPI_SWIGLU;
+    g.out = c->act;
+    g.out_ld = F;
+    g.out_hi = c->x_hi[X_FFN];
+    g.out_lo = c->x_lo[X_FFN];
+    fold_in(g);
+    return g;
+  };
+  // down projection + residual, emitting the next layer's attention RMSNorm operand (or
+  // the final RMSNorm's before the LM head)
+  auto make_down = [&](int l) {
+    GemmParams g = gemm_base(c, M, X_FFN);
+    set_plain(g, c->maps[l].down, d, F);
+    g.epi = EPI_RESID;
+    g.out = c->h;
+    g.out_ld = d;
+    fold_out(g, l + 1 < L ? c->layers[l + 1].attn_norm : c->w.final_norm);
+    return g;
+  };
+  auto make_head = [&]() {
+    GemmParams g = gemm_base(c, M, X_NORM);
+    set_plain(g, c->head_map, cf.vocab, d);
+    fold_in(g);
+    g.epi = EPI_STORE;
+    g.out = logits;
+    g.out_ld = cf.vocab;
+    return g;
+  };
+  auto gemm = [&](GemmParams& g, int cls) {
+    g.trace = next_trace(c, cls);
+    return timed(c, cls, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); });
+  };
+  if (norm(tokens, c->layers[0].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
+  GemmParams gq = make_qkv(0);
+  for (int l = 0; l < L; ++l) {
+    GemmParams go = make_o(l), gg = make_gateup(l), gd = make_down(l), gn{};
+    if (l + 1 < L) gn = make_qkv(l + 1);
+    else if (logits) gn = make_head();
+    if (gemm(gq, K_GEMM_QKV) != cudaSuccess) return SDSAT_ECUDA;
     // block-causal attention; its merge emits the O projection's operand
     AttnParams a;
     std::memset(&a, 0, sizeof(a));
@@ -301,53 +378,14 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
     a.counters = c->att_counters;
     a.err = c->err;
+    a.trace = next_trace(c, K_ATTENTION);
     if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    // O projection + residual
-    g = gemm_base(c, M, X_ATTN);
-    set_plain(g, mp.o, d, R);
-    g.epi = EPI_RESID;
-    g.out = c->h;
-    g.out_ld = d;
-    fold_out(g, c->layers[l].ffn_norm);
-    if (timed(c, K_GEMM_O, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    // gate/up with SiLU(gate) * up fused; emits the down projection's operand
-    g = gemm_base(c, M, X_NORM);
-    g.tmap[0] = mp.gate;
-    g.tmap[1] = mp.up;
-    g.map_mode = MAP_GATEUP;
-    g.N = F;
-    g.K = d;
-    g.n_tiles = (F + 63) / 64;
-    g.kc = (d + 63) / 64;
-    g.epi = EPI_SWIGLU;
-    g.out = c->act;
-    g.out_ld = F;
-    g.out_hi = c->x_hi[X_FFN];
-    g.out_lo = c->x_lo[X_FFN];
-    fold_in(g);
-    if (timed(c, K_GEMM_GATEUP, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
+    if (gemm(go, K_GEMM_O) != cudaSuccess || gemm(gg, K_GEMM_GATEUP) != cudaSuccess ||
+        gemm(gd, K_GEMM_DOWN) != cudaSuccess)
       return SDSAT_ECUDA;
-    // down projection + residual
-    g = gemm_base(c, M, X_FFN);
-    set_plain(g, mp.down, d, F);
-    g.epi = EPI_RESID;
-    g.out = c->h;
-    g.out_ld = d;
-    // the next layer's attention RMSNorm, or the final RMSNorm before the LM head
-    fold_out(g, l + 1 < L ? c->layers[l + 1].attn_norm : c->w.final_norm);
-    if (timed(c, K_GEMM_DOWN, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
-      return SDSAT_ECUDA;
+    gq = gn;
   }
-  if (logits) {
-    GemmParams g = gemm_base(c, M, X_NORM);
-    set_plain(g, c->head_map, cf.vocab, d);
-    fold_in(g);
-    g.epi = EPI_STORE;
-    g.out = logits;
-    g.out_ld = cf.vocab;
-    if (timed(c, K_GEMM_LM_HEAD, [&] { return launch_gemm(g, c->num_sms, st, c->pdl); }) != cudaSuccess)
-      return SDSAT_ECUDA;
-  }
+  if (logits && gemm(gq, K_GEMM_LM_HEAD) != cudaSuccess) return SDSAT_ECUDA;
   return SDSAT_OK;
 }
 
@@ -408,6 +446,8 @@ void sdsat_destroy(sdsat_ctx* c) {
   if (!c) return;
   cudaStreamSynchronize(c->stream);
   for (cudaEvent_t e : c->prof_events) cudaEventDestroy(e);
+  cudaFree(c->trace_rec);
+  cudaFree(c->trace_count);
   for (void* p : c->allocs) cudaFree(p);
   delete c;
 }
@@ -680,6 +720,46 @@ sdsat_status sdsat_kv_emitted(sdsat_ctx* c, sdsat_kv* kv, int64_t* emitted_dev, 
   return SDSAT_OK;
 }
 
+sdsat_status sdsat_trace_begin(sdsat_ctx* c, int max_records) {
+  if (!c || max_records < 1) return SDSAT_EINVAL;
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return SDSAT_ECUDA;
+  cudaFree(c->trace_rec);
+  cudaFree(c->trace_count);
+  c->trace_rec = nullptr;
+  c->trace_count = nullptr;
+  void *r = nullptr, *n = nullptr;
+  if (cudaMalloc(&r, (size_t)max_records * TRACE_WORDS * sizeof(unsigned long long)) != cudaSuccess) return SDSAT_ENOMEM;
+  if (cudaMalloc(&n, sizeof(unsigned int)) != cudaSuccess || cudaMemset(n, 0, sizeof(unsigned int)) != cudaSuccess) {
+    cudaFree(r);
+    return SDSAT_ENOMEM;
+  }
+  c->trace_rec = static_cast<unsigned long long*>(r);
+  c->trace_count = static_cast<unsigned int*>(n);
+  c->trace_cap = (unsigned)max_records;
+  c->trace_seq = 0;
+  return SDSAT_OK;
+}
+
+sdsat_status sdsat_trace_end(sdsat_ctx* c, uint64_t* records, int max_records, int* n_records) {
+  if (!c || !c->trace_rec) return SDSAT_EINVAL;
+  unsigned int n = 0;
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess ||
+      cudaMemcpy(&n, c->trace_count, sizeof(n), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return SDSAT_ECUDA;
+  n = std::min(n, c->trace_cap);
+  const unsigned int m = records ? std::min<unsigned int>(n, (unsigned)std::max(max_records, 0)) : 0;
+  if (m && cudaMemcpy(records, c->trace_rec, (size_t)m * TRACE_WORDS * sizeof(uint64_t), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return SDSAT_ECUDA;
+  if (n_records) *n_records = (int)m;
+  cudaFree(c->trace_rec);
+  cudaFree(c->trace_count);
+  c->trace_rec = nullptr;
+  c->trace_count = nullptr;
+  return SDSAT_OK;
+}
+
+const char* sdsat_kernel_class_name(int cls) { return (cls >= 0 && cls < K_COUNT) ? KCLASS_NAME[cls] : "?"; }
+
 sdsat_status sdsat_profile_begin(sdsat_ctx* c, int max_launches) {
   if (!c || max_launches < 1) return SDSAT_EINVAL;
   for (cudaEvent_t e : c->prof_events) cudaEventDestroy(e);
@@ -779,7 +859,8 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
     return SDSAT_EINVAL;
   AttnParams a;
   std::memset(&a, 0, sizeof(a));
-  if (!aligned16(k_dev) || !aligned16(v_dev) || (long long)b * H * cap > 0x7FFFFFFFll) return SDSAT_EINVAL;
+  if (!aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) || (long long)b * H * cap > 0x7FFFFFFFll)
+    return SDSAT_EINVAL;
   if (!make_kvmap(&a.kmap, k_dev, (long long)b * H * cap, hd) || !make_kvmap(&a.vmap, v_dev, (long long)b * H * cap, hd))
     return SDSAT_ECUDA;
   a.row0 = 0;
