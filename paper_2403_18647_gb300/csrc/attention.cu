@@ -136,6 +136,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
 
   volatile int no_abort = 0;
   bool ok = mbar_wait_bounded(&bar[0], 0, &no_abort, p.err);
+  __syncwarp();   // lanes leave the polling loop at different times: reconverge
   const unsigned long long t_k = p.trace.rec ? globaltimer_ns() : 0;
 
   // ---- S = Q K^T for this warp's 32 keys (4 tiles of 8), fp32 in registers
@@ -235,6 +236,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
 
   // ---- O = P V for this warp's HD/4 dimensions (DT tiles of 8), all 128 keys
   ok = ok && mbar_wait_bounded(&bar[1], 0, &no_abort, p.err);
+  __syncwarp();
   float O[DT][4];
 #pragma unroll
   for (int nt = 0; nt < DT; ++nt)
@@ -263,6 +265,11 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     }
   }
   const size_t prow_base = (size_t)h * p.nch_max + ch;
+  if (tid < q) {   // Ms / Ls of row tid were written by this thread; read before the stores below
+    float* ml = p.part_ml + ((size_t)(sl * q + tid) * p.H * p.nch_max + prow_base) * 2;
+    ml[0] = Ms[tid];
+    ml[1] = Ls[tid];
+  }
 #pragma unroll
   for (int nt = 0; nt < DT; ++nt)
 #pragma unroll
@@ -274,25 +281,22 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
             make_float2(O[nt][e], O[nt][e + 1]);
       }
     }
-  __syncthreads();   // Ms / Ls written
-  if (tid < q) {
-    float* ml = p.part_ml + ((size_t)(sl * q + tid) * p.H * p.nch_max + prow_base) * 2;
-    ml[0] = Ms[tid];
-    ml[1] = Ls[tid];
-  }
 
-  // the last chunk CTA of this (sequence, head) merges the chunks
+  // the last chunk CTA of this (sequence, head) merges the chunks: the CTA's stores, then
+  // one release/acquire counter update by thread 0
   const unsigned long long t_part = p.trace.rec ? globaltimer_ns() : 0;
-  __threadfence();
   __syncthreads();
-  if (tid == 0) *s_last = (atomicAdd(p.counters + sl * p.H + h, 1) == nch - 1);
+  if (tid == 0) {
+    __threadfence();
+    *s_last = (atomicAdd(p.counters + sl * p.H + h, 1) == nch - 1);
+    __threadfence();
+  }
   __syncthreads();
   if (!*s_last) {
     if (tid == 0 && p.trace.rec)
       trace_write(p.trace, (unsigned)nch << 8, t_entry, t_wait, t_k, t_part, 0, globaltimer_ns());
     return;
   }
-  __threadfence();
   // Merge weights: warp w takes rows j = w, w + 4, ...; its lanes hold the chunks.
   // w[j][c] = exp(m_c - max_c m_c) goes to shared memory (the K tile is free now),
   // 1 / L_j with L_j = sum_c w[j][c] l_c to Ms[j].

@@ -63,7 +63,7 @@ struct GemmCfg {
   static constexpr int W_BYTES = 128 * 128;      // 128 rows x 64 bf16
   static constexpr int X_BYTES = MPAD * 128;     // MPAD rows x 64 bf16 (hi or lo)
   static constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
-  static constexpr int STAGING = 128 * (MPAD + 1);
+  static constexpr int STAGING = 128 * (MPAD + 1) + 128;   // [128][MPAD+1] exchange + [128/MPAD][MPAD] sums
   static constexpr int ACC_COLS = 2 * MPAD;     // hi and lo products side by side
   static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
   static constexpr int NBAR = 2 * STAGES + 6;
@@ -107,14 +107,14 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     for (int m = 0; m < MPAD; ++m) acc[m] *= sinv[m];
   }
   if (p.epi == EPI_RESID && p.gain_next) {
-    // residual update, the next RMSNorm's operand h * g and this tile's sums of h^2
+    // Residual update h += y, the next RMSNorm's operand h * g and this tile's sums of
+    // h^2.  The sums go through shared memory in two conflict-free passes (warp shuffles
+    // measured ~0.15 us each here, serialised per row), and the global stores come last.
     const int n = 128 * tile + r;
     const bool valid = n < p.N;
-    const float gn = pre_gn;
-    const int e = r >> 5, lane = r & 31;
 #pragma unroll
     for (int m0 = 0; m0 < MPAD; m0 += EG) {
-      float hv[EG];   // a group's residual rows are loaded before anything is stored (group 0: earlier)
+      float hv[EG];
 #pragma unroll
       for (int u = 0; u < EG; ++u)
         hv[u] = m0 == 0 ? pre[u] : (m0 + u < M && valid) ? __ldcg(p.out + (size_t)(m0 + u) * p.out_ld + n) : 0.f;
@@ -122,25 +122,43 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
       for (int u = 0; u < EG; ++u) {
         const int m = m0 + u;
         if (m >= M) break;
-        float hn = 0.f;
-        if (valid) {
-          const size_t o = (size_t)m * p.out_ld + n;
-          hn = hv[u] + acc[m];
-          p.out[o] = hn;
-          const float x = hn * gn;
-          const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-          p.xn_hi[o] = hi;
-          p.xn_lo[o] = __float2bfloat16_rn(x - __bfloat162float(hi));
-        }
-        float sq = hn * hn;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-        if (lane == 0) staging[e * 64 + m] = sq;
+        acc[m] = valid ? hv[u] + acc[m] : 0.f;   // h after the update
+        staging[r * (MPAD + 1) + m] = acc[m] * acc[m];
       }
     }
     named_bar_sync(1, 128);
-    if (r < M) p.ssq_out[r * p.ssq_ld + tile] = staging[r] + staging[64 + r] + staging[128 + r] + staging[192 + r];
+    // pass 1: thread (part, m) sums lanes part*RPP .. part*RPP+RPP-1 of row m
+    constexpr int PARTS = 128 / MPAD, RPP = 128 / PARTS;   // parts of the 128 lanes, lanes per part
+    float* part_sum = staging + 128 * (MPAD + 1);          // [PARTS][MPAD], beyond the [128][MPAD+1] block
+    {
+      const int m = r % MPAD, part = r / MPAD;
+      float sq = 0.f;
+      if (m < M) {
+#pragma unroll 8
+        for (int i = 0; i < RPP; ++i) sq += staging[(part * RPP + i) * (MPAD + 1) + m];
+      }
+      part_sum[part * MPAD + m] = sq;
+    }
     named_bar_sync(1, 128);
+    float ssq = 0.f;   // pass 2: row r < M adds its parts
+    if (r < M) {
+#pragma unroll
+      for (int part = 0; part < PARTS; ++part) ssq += part_sum[part * MPAD + r];
+    }
+    named_bar_sync(1, 128);
+    if (r < M) p.ssq_out[r * p.ssq_ld + tile] = ssq;
+    if (valid) {
+#pragma unroll
+      for (int m = 0; m < MPAD; ++m) {
+        if (m >= M) break;
+        const size_t o = (size_t)m * p.out_ld + n;
+        p.out[o] = acc[m];
+        const float x = acc[m] * pre_gn;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+        p.xn_hi[o] = hi;
+        p.xn_lo[o] = __float2bfloat16_rn(x - __bfloat162float(hi));
+      }
+    }
     return;
   }
   if (p.epi == EPI_STORE || p.epi == EPI_RESID) {
@@ -170,12 +188,14 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
   if (p.epi == EPI_SWIGLU) {
     const int j = 64 * tile + r;
     if (r < 64 && j < p.N) {
+      // the up projections (lanes 64-127) leave shared memory before any store is issued
+#pragma unroll
+      for (int m = 0; m < MPAD; ++m)
+        if (m < M) acc[m] = acc[m] / (1.0f + expf(-acc[m])) * staging[(r + 64) * (MPAD + 1) + m];
 #pragma unroll
       for (int m = 0; m < MPAD; ++m) {
         if (m >= M) break;
-        const float g = acc[m];
-        const float u = staging[(r + 64) * (MPAD + 1) + m];
-        const float a = g / (1.0f + expf(-g)) * u;
+        const float a = acc[m];
         p.out[(size_t)m * p.out_ld + j] = a;
         const __nv_bfloat16 hi = __float2bfloat16_rn(a);
         p.out_hi[(size_t)m * p.out_ld + j] = hi;
@@ -192,17 +212,22 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int partner = (i < half) ? r + half : r - half;
 #pragma unroll
     for (int m0 = 0; m0 < MPAD; m0 += EG) {
-      // a group's RoPE factors first, so no load waits behind a store
+      // a group's rotated values first, then its stores (shared-memory reads queue behind stores)
       int slot[EG];
-      float2 cs[EG];
+      float val[EG];
 #pragma unroll
       for (int u = 0; u < EG; ++u) {
         const int m = m0 + u;
         slot[u] = 0;
-        cs[u] = make_float2(1.f, 0.f);
+        val[u] = 0.f;
         if (m < M) {
           slot[u] = s_slot[m];
-          if (which < 2) cs[u] = p.rope[(size_t)s_pos[m] * half + (i % half)];
+          val[u] = acc[m];
+          if (which < 2) {   // rotate-half RoPE with the partner lane's value from shared memory
+            const float2 cs = p.rope[(size_t)s_pos[m] * half + (i % half)];
+            const float y = staging[partner * (MPAD + 1) + m];
+            val[u] = (i < half) ? acc[m] * cs.x - y * cs.y : acc[m] * cs.x + y * cs.y;
+          }
         }
       }
 #pragma unroll
@@ -210,17 +235,11 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
         const int m = m0 + u;
         if (m >= M) break;
         const int s = p.seq0 + m / p.q;
-        const float x = acc[m];
-        float val = x;
-        if (which < 2) {
-          const float y = staging[partner * (MPAD + 1) + m];
-          val = (i < half) ? x * cs[u].x - y * cs[u].y : x * cs[u].x + y * cs[u].y;
-        }
         if (which == 0) {
-          p.out[(size_t)m * p.out_ld + f] = val;
+          p.out[(size_t)m * p.out_ld + f] = val[u];
         } else if (slot[u] < p.cap) {
           __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
-          cache[(((size_t)s * p.H + head) * p.cap + slot[u]) * hd + i] = __float2bfloat16_rn(val);
+          cache[(((size_t)s * p.H + head) * p.cap + slot[u]) * hd + i] = __float2bfloat16_rn(val[u]);
         } else if (i == 0 && which == 1) {
           set_error(p.err, ERR_CAPACITY);
         }
@@ -418,7 +437,9 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
         if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
       }
-      if (!mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err)) break;
+      const bool got = mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err);
+      __syncwarp();   // lanes leave the polling loop at different times: reconverge
+      if (!got) break;
       tc_fence_after();
       const bool last_seg = g >= g1;
       if (r == 0 && last_seg && p.trace.rec) s_mark[1] = globaltimer_ns();
@@ -486,6 +507,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
               }
             }
             ok = mbar_wait_bounded(red_bar, ph, abort_flag, p.err);
+            __syncwarp();
             ph ^= 1u;
             if (ok) {
               for (int u = 0; u < cnt; ++u) {
