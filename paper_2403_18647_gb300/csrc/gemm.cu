@@ -36,18 +36,17 @@ namespace sdsat {
 
 // Pipeline depth and CTAs per SM (compile-time tuning).  Measured on GB300: one CTA
 // per SM streams ~5 TB/s whatever its depth (3..10 stages), two CTAs per SM ~7 TB/s.
-// For M <= 16 two 3-stage CTAs (~71 KB of shared memory each) run per SM, which
-// still leaves room for one CTA of the next kernel to start prefetching its weights.
+// For M <= 16 a CTA has 4 stages (~91 KB of shared memory), so exactly two fit on an
+// SM.  With 3 stages (~71 KB) a third fits: the next kernel's CTAs then start early,
+// but the scheduler also stacks three CTAs of one GEMM on some SMs and one on others,
+// and the equal stream-K shares finish unevenly (7B step 3.80 ms vs 3.70 with 4).
 #ifndef SDSAT_GEMM_STAGES16
-#define SDSAT_GEMM_STAGES16 3
+#define SDSAT_GEMM_STAGES16 4
 #endif
 #ifndef SDSAT_GEMM_CTAS_PER_SM
 #define SDSAT_GEMM_CTAS_PER_SM 2
 #endif
 // Minimum resident CTAs per SM the register allocation must allow (192 threads each).
-// The M <= 16 kernel stays below 112 registers without it (-Xptxas -v), so a third CTA
-// -- the next kernel's, launched early by programmatic dependent launch -- fits beside
-// two running ones and prefetches its weights.
 #ifndef SDSAT_GEMM_MINB
 #define SDSAT_GEMM_MINB 2
 #endif
@@ -495,16 +494,14 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
           bool ok = true;
           for (int j0 = c_lo; j0 <= c_hi && ok; j0 += per) {
             const int cnt = min(per, c_hi - j0 + 1);
-            named_bar_sync(1, 128);   // the previous round's shared-memory reads are done
-            if (r == 0) {
+            if (r == 0) mbar_arrive_expect_tx(red_bar, (uint32_t)cnt * pbytes);
+            named_bar_sync(1, 128);   // the previous round's shared-memory reads are done; bytes announced
+            if (r < cnt) {            // one copy per thread
+              const int j = j0 + r;
+              const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
               fence_proxy_async_global();
-              mbar_arrive_expect_tx(red_bar, (uint32_t)cnt * pbytes);
-              for (int u = 0; u < cnt; ++u) {
-                const int j = j0 + u;
-                const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
-                bulk_load_g2s(stages + (size_t)u * pbytes,
-                              p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128, pbytes, red_bar);
-              }
+              bulk_load_g2s(stages + (size_t)r * pbytes,
+                            p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128, pbytes, red_bar);
             }
             ok = mbar_wait_bounded(red_bar, ph, abort_flag, p.err);
             __syncwarp();

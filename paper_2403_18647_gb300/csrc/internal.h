@@ -106,11 +106,12 @@ cudaError_t gemm_prepare();           // set smem attributes (idempotent)
 cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl);
 
 // ---- attention -------------------------------------------------------------
-constexpr int ATT_CHUNK = 128;
-constexpr int ATT_MAX_CHUNKS = 256;   // contexts up to 32768 slots (the merge keeps q x chunks stats in smem)
+constexpr int ATT_UNIT = 64;          // keys per work unit: one TMA box of cache rows
+constexpr int ATT_MAX_CAP = 32768;    // KV capacity (slots per sequence) the kernel supports
+constexpr int ATT_SEG_MAX = 16;       // CTAs that may share one (sequence, head): partial slots per pair
 #define SDSAT_ATT_MAXQ 16
 struct AttnParams {
-  CUtensorMap kmap;     // the K cache as a 2-D tensor [rows][hd] bf16, boxes of 64 dims x ATT_CHUNK rows
+  CUtensorMap kmap;     // the K cache as a 2-D tensor [rows][hd] bf16, boxes of 64 dims x ATT_UNIT rows
   CUtensorMap vmap;     // the V cache, same geometry
   int row0;             // first row of this layer: cache row of (s, h, slot) = row0 + (s*H + h)*cap + slot
   const float* Q;       // [rows][q_ld] (row = sl*q + j), head h at column h*hd
@@ -121,15 +122,16 @@ struct AttnParams {
   int out_ld;
   __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
   __nv_bfloat16* out_lo;
-  float* part_o;        // [rows][H][nch_max][hd]
-  float* part_ml;       // [rows][H][nch_max][2]
-  int nch_max;
-  int* counters;        // [nb][H]
+  float* part_o;        // [rows][H][ATT_SEG_MAX][hd]: one unnormalised partial output per CTA sharing a pair
+  float* part_ml;       // [rows][H][ATT_SEG_MAX][2]: its running max and exp-sum
+  int* counters;        // [nb][H], zero between launches
   uint32_t* err;
   Trace trace;
 };
+size_t attention_smem_bytes(int hd);
 cudaError_t attention_prepare();   // set smem attributes (idempotent)
-cudaError_t launch_attention(const AttnParams& p, cudaStream_t st, bool pdl);
+// grid: min(2 * num_sms, 14 * H) CTAs, so at most ATT_SEG_MAX CTAs share one (sequence, head)
+cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl);
 
 // ---- embedding, acceptance, block building ------------------------------------
 // x = h * rsqrt(mean h^2 + eps) * g, stored as bf16 hi + lo (tokens != null: h = E[tokens] first)

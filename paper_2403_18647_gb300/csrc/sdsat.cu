@@ -63,12 +63,12 @@ bool make_xmap(CUtensorMap* map, const void* ptr, int rows, int cols, int box_ro
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// bf16 KV cache viewed as [rows][hd], boxes of 64 dims x ATT_CHUNK rows, 128-byte swizzle
+// bf16 KV cache viewed as [rows][hd], boxes of 64 dims x ATT_UNIT rows, 128-byte swizzle
 bool make_kvmap(CUtensorMap* map, const void* ptr, long long rows, int hd) {
   if (!get_encode()) return false;
   cuuint64_t dims[2] = {(cuuint64_t)hd, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
-  cuuint32_t box[2] = {64, (cuuint32_t)ATT_CHUNK};
+  cuuint32_t box[2] = {64, (cuuint32_t)ATT_UNIT};
   cuuint32_t estr[2] = {1, 1};
   return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -122,7 +122,6 @@ struct sdsat_ctx {
   int ssq_ld = 0;
   float* att_part_o = nullptr;
   float* att_part_ml = nullptr;
-  int att_nch = 0;
   int* att_counters = nullptr;
   int* acc_targets = nullptr;
   int* acc_counters = nullptr;
@@ -375,11 +374,11 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.out_lo = c->x_lo[X_ATTN];
     a.part_o = c->att_part_o;
     a.part_ml = c->att_part_ml;
-    a.nch_max = std::min(c->att_nch, (kv->cap + ATT_CHUNK - 1) / ATT_CHUNK);
     a.counters = c->att_counters;
     a.err = c->err;
     a.trace = next_trace(c, K_ATTENTION);
-    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, c->num_sms, st, c->pdl); }) != cudaSuccess)
+      return SDSAT_ECUDA;
     if (gemm(go, K_GEMM_O) != cudaSuccess || gemm(gg, K_GEMM_GATEUP) != cudaSuccess ||
         gemm(gd, K_GEMM_DOWN) != cudaSuccess)
       return SDSAT_ECUDA;
@@ -511,14 +510,13 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
       rope[(size_t)p * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
     }
   const int rows = SDSAT_MAX_ROWS;
-  c->att_nch = (cfg->max_position + ATT_CHUNK - 1) / ATT_CHUNK;
   c->ssq_ld = (d + 127) / 128;
   bool ok = dalloc(c, &c->rope, rope.size()) && dalloc(c, &c->h, (size_t)rows * d) &&
             dalloc(c, &c->qbuf, (size_t)rows * R) && dalloc(c, &c->attn, (size_t)rows * R) &&
             dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 2 * 64 * 128) &&
             dalloc(c, &c->gemm_counters, MAX_GEMM_TILES) &&
-            dalloc(c, &c->att_part_o, (size_t)rows * cfg->n_heads * c->att_nch * cfg->head_dim) &&
-            dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * c->att_nch * 2) &&
+            dalloc(c, &c->att_part_o, (size_t)rows * cfg->n_heads * ATT_SEG_MAX * cfg->head_dim) &&
+            dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * ATT_SEG_MAX * 2) &&
             dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
             dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)rows * OP_MAX_K) &&
@@ -557,7 +555,7 @@ sdsat_status sdsat_set_stream(sdsat_ctx* c, void* stream) {
 sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** out) {
   if (!c || !out || batch < 1 || max_len < 1) return SDSAT_EINVAL;
   *out = nullptr;
-  if (max_len > c->cfg.max_position || max_len > ATT_CHUNK * ATT_MAX_CHUNKS) return SDSAT_ECAPACITY;
+  if (max_len > c->cfg.max_position || max_len > ATT_MAX_CAP) return SDSAT_ECAPACITY;
   sdsat_kv* kv = new (std::nothrow) sdsat_kv();
   if (!kv) return SDSAT_ENOMEM;
   kv->ctx = c;
@@ -849,12 +847,11 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
                                 const int32_t* len_dev, int b, int q, int H, int hd, int cap, float* out_dev) {
   if (!c || !q_dev || !k_dev || !v_dev || !len_dev || !out_dev) return SDSAT_EINVAL;
   if (b < 1 || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS || (hd != 64 && hd != 128) || H < 1 || cap < 1 ||
-      cap > ATT_CHUNK * ATT_MAX_CHUNKS)
+      cap > ATT_MAX_CAP)
     return SDSAT_EINVAL;
-  // the split-KV workspace was sized at create for SDSAT_MAX_ROWS rows of the model's heads
-  const size_t nch = (size_t)(cap + ATT_CHUNK - 1) / ATT_CHUNK;
-  const size_t have = (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * c->att_nch;
-  if ((size_t)b * q * H * nch * hd > have * c->cfg.head_dim || (size_t)b * q * H * nch > have ||
+  // the partial-result workspace was sized at create for SDSAT_MAX_ROWS rows of the model's heads
+  const size_t have = (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * ATT_SEG_MAX;
+  if ((size_t)b * q * H * ATT_SEG_MAX * hd > have * c->cfg.head_dim || (size_t)b * q * H * ATT_SEG_MAX > have ||
       (size_t)b * H > (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads)
     return SDSAT_EINVAL;
   AttnParams a;
@@ -880,10 +877,10 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   a.out_lo = c->x_lo[X_ATTN];
   a.part_o = c->att_part_o;
   a.part_ml = c->att_part_ml;
-  a.nch_max = (cap + ATT_CHUNK - 1) / ATT_CHUNK;
   a.counters = c->att_counters;
   a.err = c->err;
-  return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->stream, c->pdl); }) == cudaSuccess ? SDSAT_OK
+  return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->num_sms, c->stream, c->pdl); }) == cudaSuccess
+             ? SDSAT_OK
                                                                                                    : SDSAT_ECUDA;
 }
 
