@@ -49,6 +49,14 @@ WORKLOADS = {
 }
 
 
+# DRAM bytes (read + write) per algorithmic byte of the skinny GEMM, from one ncu capture
+# (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.35 MB of traffic for
+# 181.0 MB of weights + operand + output.  Applied to the average launch of the step.
+GEMM_TRAFFIC_RATIO = 186.35 / 181.0
+GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.35 MB for 181.0 MB "
+                       "algorithmic), ratio scaled to the average launch; bytes per launch")
+
+
 def expected_tokens_per_step(k: int, match: float) -> float:
     """Two steps emit 2 + m tokens, m = leading matches of k drafts (Sec. 2.1.1)."""
     return (2.0 + sum(match ** j for j in range(1, k + 1))) / 2.0
@@ -370,7 +378,9 @@ def run_ours(args, wl, rank, world):
                      "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4),
                      "frac_of_measured": round(step_gbs / peak, 4)},
         "roofline": {"kernel": "skinny_gemm (all projections)", "bound": "hbm", "achieved": round(achieved, 1),
-                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": int(GEMM_TRAFFIC_RATIO * g_bytes / max(1, g_launches)),
+                     "traffic_source": GEMM_TRAFFIC_SOURCE,
                      "peak_source": peak_kind, "launches": g_launches,
                      "bytes_per_launch": int(g_bytes / max(1, g_launches)),
                      "ms_per_launch": round(g_ms / max(1, g_launches), 5)},

@@ -12,7 +12,8 @@
 // contiguous range [iU/P, (i+1)U/P): every CTA streams the same number of
 // K/V bytes.  One thread keeps a two-stage ring of K and V tiles (TMA, boxes
 // of 64 dims x 64 rows, 128-byte swizzle) full; tiles made of committed slots
-// only are requested before the QKV projection has finished.  Per unit, on
+// only are requested before the QKV projection has finished, and the next
+// ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on
 // the tensor cores (mma.sync m16n8k16, the q <= 16 rows fill the M = 16
 // tile): S = Q K^T with each warp on 16 keys, an online-softmax update of the
 // running row max and exp-sum (row reductions through shared memory), then
@@ -33,6 +34,7 @@
 namespace sdsat {
 
 constexpr int ATT_STAGES = 2;
+constexpr int ATT_PREFETCH = 4;   // units past the ring requested into L2 ahead of their loads
 
 template <int HD>
 struct AttCfg {
@@ -185,15 +187,15 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     tma_prefetch_desc(&p.vmap);
     pol = l2_policy_evict_first();
     // Tiles of committed slots do not depend on the QKV projection: the first ones go
-    // to the ring now, the rest of the range into L2, so that the ring's later loads
-    // are L2 hits instead of one HBM round trip per unit.
+    // to the ring now, the next ATT_PREFETCH into L2 (and one more each time the ring is
+    // refilled), so that the ring's loads are L2 hits instead of HBM round trips.
     for (; issued < min(n, ATT_STAGES); ++issued) {
       bool committed;
       const int row = unit_row(u0 + issued, committed);
       if (!committed) break;
       issue(issued, row);
     }
-    for (int k = ATT_STAGES; k < n; ++k) {
+    for (int k = ATT_STAGES; k < min(n, ATT_STAGES + ATT_PREFETCH); ++k) {
       bool committed;
       const int row = unit_row(u0 + k, committed);
       if (committed) prefetch(row);
@@ -213,7 +215,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   const float scale = rsqrtf((float)HD);
   const int kb = warp * 16;                       // first key (within the unit) of this warp's scores
   const int db = warp * (HD / 4);                 // first dimension of this warp's outputs
-  float O[DT][4];
+  float O[DT][4], Ol[DT][4];   // P.V with the hi and with the lo part of P, summed when published
   int sl = 0, h = 0, c = 0;
   locate(u0, sl, h, c);
   int seg_first = u0;                             // first unit of the current (sequence, head) run
@@ -242,7 +244,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
 #pragma unroll
       for (int nt = 0; nt < DT; ++nt)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) O[nt][e] = 0.f;
+        for (int e = 0; e < 4; ++e) O[nt][e] = Ol[nt][e] = 0.f;
       __syncthreads();
     }
     const int len = len_seq[sl];
@@ -344,6 +346,10 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
         O[nt][1] *= a0;
         O[nt][2] *= a1;
         O[nt][3] *= a1;
+        Ol[nt][0] *= a0;
+        Ol[nt][1] *= a0;
+        Ol[nt][2] *= a1;
+        Ol[nt][3] *= a1;
       }
     }
     if (ok) {
@@ -361,16 +367,17 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
           uint32_t b0, b1, b2, b3;
           ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), b0, b1, b2, b3);
           mma_bf16_16816(O[2 * np], ah[0], ah[1], ah[2], ah[3], b0, b1);
-          mma_bf16_16816(O[2 * np], al[0], al[1], al[2], al[3], b0, b1);
+          mma_bf16_16816(Ol[2 * np], al[0], al[1], al[2], al[3], b0, b1);
           mma_bf16_16816(O[2 * np + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-          mma_bf16_16816(O[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
+          mma_bf16_16816(Ol[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
         }
       }
     }
     __syncthreads();   // the stage, P and the row statistics are consumed
-    if (tid == 0 && issued < n && !*abort_flag) {   // refill the freed stage
+    if (tid == 0 && issued < n && !*abort_flag) {   // refill the freed stage, extend the L2 window
       bool committed;
       issue(issued, unit_row(u0 + issued, committed));
+      if (issued + ATT_PREFETCH < n) prefetch(unit_row(u0 + issued + ATT_PREFETCH, committed));
       ++issued;
     }
 
@@ -396,7 +403,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
           if (j < q && fits) {
             const int dim = db + 8 * nt + 2 * tig;
             *reinterpret_cast<float2*>(p.part_o + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * HD + dim) =
-                make_float2(O[nt][e], O[nt][e + 1]);
+                make_float2(O[nt][e] + Ol[nt][e], O[nt][e + 1] + Ol[nt][e + 1]);
           }
         }
       if (p.trace.rec) t_part = globaltimer_ns();

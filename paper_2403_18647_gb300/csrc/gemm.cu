@@ -58,7 +58,7 @@ constexpr int EG = SDSAT_GEMM_EPI_GROUP;
 
 template <int MPAD>
 struct GemmCfg {
-  static constexpr int STAGES = MPAD <= 16 ? SDSAT_GEMM_STAGES16 : (MPAD <= 32 ? 4 : 3);
+  static constexpr int STAGES = MPAD <= 16 ? SDSAT_GEMM_STAGES16 : 3;   // M <= 32: two CTAs per SM
   static constexpr int W_BYTES = 128 * 128;      // 128 rows x 64 bf16
   static constexpr int X_BYTES = MPAD * 128;     // MPAD rows x 64 bf16 (hi or lo)
   static constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
@@ -99,7 +99,8 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
                                                float* staging, const float* sinv, const int* s_slot,
-                                               const int* s_pos, const float (&pre)[EG], float pre_gn) {
+                                               const int* s_pos, const float (&pre)[EG], float pre_gn,
+                                               const float2 (&pre_cs)[EG]) {
   const int M = p.M;
   if (p.ssq_in) {
 #pragma unroll
@@ -223,7 +224,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
           slot[u] = s_slot[m];
           val[u] = acc[m];
           if (which < 2) {   // rotate-half RoPE with the partner lane's value from shared memory
-            const float2 cs = p.rope[(size_t)s_pos[m] * half + (i % half)];
+            const float2 cs = m0 == 0 ? pre_cs[u] : p.rope[(size_t)s_pos[m] * half + (i % half)];
             const float y = staging[partner * (MPAD + 1) + m];
             val[u] = (i < half) ? acc[m] * cs.x - y * cs.y : acc[m] * cs.x + y * cs.y;
           }
@@ -425,16 +426,22 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
       const int tile = (int)(g / p.kc);
       g = std::min(g1, (long long)(tile + 1) * p.kc);
       const int buf = seg & 1;
-      // the residual rows (first group) and gain this tile's epilogue needs, loaded while
-      // the tensor cores work
+      // what this tile's epilogue reads from global memory (first row group), loaded while
+      // the tensor cores work: residual rows and gain, or RoPE factors
       float pre[EG];
       float pre_gn = 0.f;
+      float2 pre_cs[EG];
       {
         const int n = 128 * tile + r;
         const bool resid = p.epi == EPI_RESID && n < p.N;
 #pragma unroll
         for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
         if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
+        const bool rope = p.epi == EPI_QKV && n / p.rows_per_map < 2;   // a q or k feature (rows_per_map > 0)
+        const int half = max(p.hd >> 1, 1), ih = rope ? (n % p.rows_per_map) % p.hd % half : 0;
+#pragma unroll
+        for (int u = 0; u < EG; ++u)
+          pre_cs[u] = (rope && u < p.M) ? p.rope[(size_t)s_pos[u] * half + ih] : make_float2(1.f, 0.f);
       }
       const bool got = mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err);
       __syncwarp();   // lanes leave the polling loop at different times: reconverge
@@ -529,7 +536,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         if (r == 0) p.counters[tile] = 0;
       }
       if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
-      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn);
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn, pre_cs);
     }
   }
 
@@ -562,7 +569,7 @@ cudaError_t gemm_prepare() {
 
 static int gemm_grid(const GemmParams& p, int num_sms) {
   const long long T = (long long)p.n_tiles * p.kc;
-  const int per_sm = gemm_mpad(p.M) <= 16 ? SDSAT_GEMM_CTAS_PER_SM : 1;
+  const int per_sm = gemm_mpad(p.M) <= 32 ? SDSAT_GEMM_CTAS_PER_SM : 1;
   return (int)std::min<long long>((long long)num_sms * per_sm, T);
 }
 
