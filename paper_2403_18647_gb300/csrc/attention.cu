@@ -13,13 +13,14 @@
 // K/V bytes.  One thread keeps a two-stage ring of K and V tiles (TMA, boxes
 // of 64 dims x 64 rows, 128-byte swizzle) full; tiles made of committed slots
 // only are requested before the QKV projection has finished, and the next
-// ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on
-// the tensor cores (mma.sync m16n8k16, the q <= 16 rows fill the M = 16
-// tile): S = Q K^T with each warp on 16 keys, an online-softmax update of the
-// running row max and exp-sum (row reductions through shared memory), then
-// O = O * alpha + P V with each warp on hd/4 dimensions.  Q and P enter as
-// bf16 hi + lo pairs (two MMAs each), K and V are the cache's own bf16
-// values, accumulation is fp32.
+// ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on the tensor
+// cores (mma.sync m16n8k16) in transposed form, so that the q <= 8 block rows
+// fill an N = 8 tile instead of padding an M = 16 one: S^T = K Q^T with each
+// warp on 16 keys, an online-softmax update of the running row max and
+// exp-sum (reductions over the warp's lanes, then the warps via shared
+// memory), then O^T = O^T * alpha + V^T P^T with each warp on hd/4
+// dimensions.  Q and P enter as bf16 hi + lo pairs (two MMAs each), K and V
+// are the cache's own bf16 values, accumulation is fp32.
 //
 // A CTA's run of units of one (sequence, head) ends in a partial result (row
 // max, exp-sum, unnormalised output).  The last of the <= ATT_SEG_MAX CTAs
@@ -48,8 +49,7 @@ struct AttCfg {
   static constexpr size_t OFF_Q = (size_t)ATT_STAGES * STAGE;
   static constexpr size_t OFF_P = OFF_Q + 2 * 16 * QSTRIDE;
   static constexpr size_t OFF_RED = OFF_P + 2 * 16 * PSTRIDE;                       // [16][RED]
-  static constexpr size_t OFF_ROW = OFF_RED + 16 * RED * 4;                         // m, l, alpha [16]
-  static constexpr size_t OFF_MERGE = OFF_ROW + 3 * 16 * 4;                         // ms, ls, w [16][SEG], inv [16]
+  static constexpr size_t OFF_MERGE = OFF_RED + 16 * RED * 4;                       // ms, ls, w [16][SEG], inv [16]
   static constexpr size_t OFF_SEQ = OFF_MERGE + (3 * 16 * ATT_SEG_MAX + 16) * 4;    // len, units [64], first unit [65]
   static constexpr size_t OFF_BAR = (OFF_SEQ + (64 + 64 + 65) * 4 + 7) / 8 * 8;
   static constexpr size_t SMEM = 1024 + OFF_BAR + ATT_STAGES * 8 + 16;
@@ -84,11 +84,12 @@ __device__ __forceinline__ int att_cta_of(int u, int U, int P) {
   return (int)(((long long)(u + 1) * P - 1) / U);
 }
 
-template <int HD>
+// QT: tiles of 8 query rows (1 for q <= 8, 2 for q <= 16)
+template <int HD, int QT>
 __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ AttnParams p) {
   using C = AttCfg<HD>;
   constexpr int KSTEPS = HD / 16;          // MMA k-steps over the head dimension
-  constexpr int DT = HD / 32;              // 8-wide dimension tiles per warp in P.V
+  constexpr int MT = HD / 64;              // 16-dimension tiles per warp in V^T P^T
   constexpr int D4 = HD / 4;               // float4 columns of an output row
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -96,10 +97,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   uint8_t* Ql = Qh + 16 * C::QSTRIDE;               // lo part
   uint8_t* Ph = smem + C::OFF_P;                    // bf16 [16][ATT_UNIT] softmax numerators, hi part
   uint8_t* Pl = Ph + 16 * C::PSTRIDE;
-  float* red = reinterpret_cast<float*>(smem + C::OFF_RED);     // [16 rows][RED]: one value per (warp, quad lane)
-  float* m_run = reinterpret_cast<float*>(smem + C::OFF_ROW);   // [16] running row max
-  float* l_run = m_run + 16;                                    // [16] running exp-sum
-  float* alpha = l_run + 16;                                    // [16] rescale of the units before
+  float* red = reinterpret_cast<float*>(smem + C::OFF_RED);     // row-reduction scratch
   float* ms = reinterpret_cast<float*>(smem + C::OFF_MERGE);    // [16][ATT_SEG_MAX] partial maxima
   float* ls = ms + 16 * ATT_SEG_MAX;                            // partial exp-sums
   float* wg = ls + 16 * ATT_SEG_MAX;                            // merge weights
@@ -215,7 +213,13 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   const float scale = rsqrtf((float)HD);
   const int kb = warp * 16;                       // first key (within the unit) of this warp's scores
   const int db = warp * (HD / 4);                 // first dimension of this warp's outputs
-  float O[DT][4], Ol[DT][4];   // P.V with the hi and with the lo part of P, summed when published
+  // O^T of this warp's HD/4 dimensions (MT tiles of 16) x the query tiles, products with the
+  // hi and with the lo part of P (summed when published); this thread holds query rows
+  // t*8 + 2*tig + {0, 1} and keeps their running max and exp-sum in registers
+  float O[MT][QT][4], Ol[MT][QT][4];
+  float mr[QT][2], lr[QT][2];
+#pragma unroll
+  for (int t = 0; t < QT; ++t) mr[t][0] = mr[t][1] = -INFINITY, lr[t][0] = lr[t][1] = 0.f;
   int sl = 0, h = 0, c = 0;
   locate(u0, sl, h, c);
   int seg_first = u0;                             // first unit of the current (sequence, head) run
@@ -237,14 +241,14 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
         *reinterpret_cast<uint32_t*>(Ql + j * C::QSTRIDE + d * 2) =
             pack_bf16(x0 - __bfloat162float(h0), x1 - __bfloat162float(h1));
       }
-      if (tid < 16) {
-        m_run[tid] = -INFINITY;
-        l_run[tid] = 0.f;
-      }
 #pragma unroll
-      for (int nt = 0; nt < DT; ++nt)
+      for (int t = 0; t < QT; ++t) mr[t][0] = mr[t][1] = -INFINITY, lr[t][0] = lr[t][1] = 0.f;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) O[nt][e] = Ol[nt][e] = 0.f;
+      for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int t = 0; t < QT; ++t)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) O[mt][t][e] = Ol[mt][t][e] = 0.f;
       __syncthreads();
     }
     const int len = len_seq[sl];
@@ -256,120 +260,140 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     __syncwarp();   // lanes leave the polling loop at different times: reconverge
     if (k == 0 && p.trace.rec) t_k = globaltimer_ns();
 
-    // ---- S = Q K^T for this warp's 16 keys (2 tiles of 8), fp32 in registers
-    float S[2][4], Sl[2][4];   // products with the hi and the lo part of q, summed after the loop
+    // ---- S^T = K Q^T for this warp's 16 keys: m16n8k16 with A = K (16 keys x 16 dims) and
+    // B = Q^T (16 dims x 8 query rows), so up to 8 block rows fill one N = 8 tile
+    float St[QT][4], Sl[QT][4];   // products with the hi and the lo part of q
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
+    for (int t = 0; t < QT; ++t)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) S[nt][e] = Sl[nt][e] = 0.f;
+      for (int e = 0; e < 4; ++e) St[t][e] = Sl[t][e] = 0.f;
     if (ok) {
 #pragma unroll
       for (int kk = 0; kk < KSTEPS; ++kk) {
-        uint32_t ah[4], al[4];
-        const int qrow = r8 + 8 * (mi & 1), qcol = kk * 16 + 8 * (mi >> 1);
-        ldsm_x4(smem_u32(Qh + qrow * C::QSTRIDE + qcol * 2), ah[0], ah[1], ah[2], ah[3]);
-        ldsm_x4(smem_u32(Ql + qrow * C::QSTRIDE + qcol * 2), al[0], al[1], al[2], al[3]);
         const int hh = kk >> 2, cg = 2 * (kk & 3);  // 64-dim half and first 16-byte granule
-        const int key = kb + 8 * (mi >> 1) + r8;
-        const int cc = cg + (mi & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(smem_u32(Kt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), b0, b1, b2, b3);
-        mma_bf16_16816(S[0], ah[0], ah[1], ah[2], ah[3], b0, b1);
-        mma_bf16_16816(Sl[0], al[0], al[1], al[2], al[3], b0, b1);
-        mma_bf16_16816(S[1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-        mma_bf16_16816(Sl[1], al[0], al[1], al[2], al[3], b2, b3);
+        const int key = kb + r8 + 8 * (mi & 1), cc = cg + (mi >> 1);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(smem_u32(Kt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), a0, a1, a2, a3);
+#pragma unroll
+        for (int t = 0; t < QT; ++t) {
+          uint32_t bh0, bh1, bl0, bl1;   // q rows t*8 .. t*8+7: hi (matrices 0, 1), lo (2, 3)
+          const uint8_t* qsrc = (mi >> 1) ? Ql : Qh;
+          ldsm_x4(smem_u32(qsrc + (t * 8 + r8) * C::QSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), bh0, bh1, bl0, bl1);
+          mma_bf16_16816(St[t], a0, a1, a2, a3, bh0, bh1);
+          mma_bf16_16816(Sl[t], a0, a1, a2, a3, bl0, bl1);
+        }
       }
 #pragma unroll
-      for (int nt = 0; nt < 2; ++nt)
+      for (int t = 0; t < QT; ++t)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) S[nt][e] += Sl[nt][e];
+        for (int e = 0; e < 4; ++e) St[t][e] += Sl[t][e];
     }
+    // St[t][e] is the score of key kb + g + 8*(e >> 1) for query row t*8 + 2*tig + (e & 1).
     // mask: row j sees key slot kp iff kp <= len + j (and kp < nkeys, j < q)
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
+    for (int t = 0; t < QT; ++t)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        const int j = g + 8 * (e >> 1);
-        const int kp = c0 + kb + 8 * nt + 2 * tig + (e & 1);
-        if (!ok || j >= q || kp >= nkeys || kp > len + j) S[nt][e] = -INFINITY;
+        const int j = t * 8 + 2 * tig + (e & 1);
+        const int kp = c0 + kb + g + 8 * (e >> 1);
+        if (!ok || j >= q || kp >= nkeys || kp > len + j) St[t][e] = -INFINITY;
       }
-    // ---- the unit's row max -> running max, and the rescale of the units before
-    red[g * C::RED + warp * 4 + tig] = fmaxf(fmaxf(S[0][0], S[0][1]), fmaxf(S[1][0], S[1][1]));
-    red[(g + 8) * C::RED + warp * 4 + tig] = fmaxf(fmaxf(S[0][2], S[0][3]), fmaxf(S[1][2], S[1][3]));
-    __syncthreads();
-    if (tid < 16) {
-      float mc = -INFINITY;
+    // ---- the unit's row maxima: over the warp's lanes holding other keys (g), then the four
+    // warps through shared memory; the running statistics stay in registers
+    float* redm = red;          // [4 warps][16 rows] unit row maxima
+    float* redl = red + 64;     // [4 warps][16 rows] unit row exp-sums
+    float mx[QT][2];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) mc = fmaxf(mc, red[tid * C::RED + i]);
-      const float mo = m_run[tid], mn = fmaxf(mo, mc);
-      alpha[tid] = (mn == -INFINITY) ? 1.f : expf(mo - mn);
-      m_run[tid] = mn;
+    for (int t = 0; t < QT; ++t) {
+      mx[t][0] = fmaxf(St[t][0], St[t][2]);
+      mx[t][1] = fmaxf(St[t][1], St[t][3]);
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        mx[t][0] = fmaxf(mx[t][0], __shfl_xor_sync(0xffffffffu, mx[t][0], o));
+        mx[t][1] = fmaxf(mx[t][1], __shfl_xor_sync(0xffffffffu, mx[t][1], o));
+      }
+      if (g == 0) {
+        redm[warp * 16 + t * 8 + 2 * tig] = mx[t][0];
+        redm[warp * 16 + t * 8 + 2 * tig + 1] = mx[t][1];
+      }
     }
     __syncthreads();
-    // ---- P = exp(S - m) as bf16 hi + lo, and its row sums
-    const float mr0 = m_run[g], mr1 = m_run[g + 8];
-    float l0 = 0.f, l1 = 0.f;
+    float al[QT][2];   // rescale of what the units before contributed
 #pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      float pv[4];
+    for (int t = 0; t < QT; ++t)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) pv[e] = (S[nt][e] == -INFINITY) ? 0.f : expf(S[nt][e] - ((e < 2) ? mr0 : mr1));
-      l0 += pv[0] + pv[1];
-      l1 += pv[2] + pv[3];
-      const int key = kb + 8 * nt + 2 * tig;
-      const __nv_bfloat16 h0 = __float2bfloat16_rn(pv[0]), h1 = __float2bfloat16_rn(pv[1]);
-      const __nv_bfloat16 h2 = __float2bfloat16_rn(pv[2]), h3 = __float2bfloat16_rn(pv[3]);
-      *reinterpret_cast<uint32_t*>(Ph + g * C::PSTRIDE + key * 2) =
-          (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-      *reinterpret_cast<uint32_t*>(Ph + (g + 8) * C::PSTRIDE + key * 2) =
-          (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
-      *reinterpret_cast<uint32_t*>(Pl + g * C::PSTRIDE + key * 2) =
-          pack_bf16(pv[0] - __bfloat162float(h0), pv[1] - __bfloat162float(h1));
-      *reinterpret_cast<uint32_t*>(Pl + (g + 8) * C::PSTRIDE + key * 2) =
-          pack_bf16(pv[2] - __bfloat162float(h2), pv[3] - __bfloat162float(h3));
+      for (int i = 0; i < 2; ++i) {
+        const int j = t * 8 + 2 * tig + i;
+        const float mc = fmaxf(fmaxf(redm[j], redm[16 + j]), fmaxf(redm[32 + j], redm[48 + j]));
+        const float mn = fmaxf(mr[t][i], mc);
+        al[t][i] = (mn == -INFINITY) ? 1.f : __expf(mr[t][i] - mn);
+        mr[t][i] = mn;
+      }
+    // ---- P^T = exp(S^T - m) as bf16 hi + lo, stored as P [query row][key], and its row sums
+    float rs[QT][2];   // this thread's part of the unit row sums
+#pragma unroll
+    for (int t = 0; t < QT; ++t) {
+      rs[t][0] = rs[t][1] = 0.f;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int i = e & 1, j = t * 8 + 2 * tig + i, key = kb + g + 8 * (e >> 1);
+        const float pv = (St[t][e] == -INFINITY) ? 0.f : __expf(St[t][e] - mr[t][i]);
+        rs[t][i] += pv;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(pv);
+        *reinterpret_cast<__nv_bfloat16*>(Ph + j * C::PSTRIDE + key * 2) = hi;
+        *reinterpret_cast<__nv_bfloat16*>(Pl + j * C::PSTRIDE + key * 2) = __float2bfloat16_rn(pv - __bfloat162float(hi));
+      }
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        rs[t][0] += __shfl_xor_sync(0xffffffffu, rs[t][0], o);
+        rs[t][1] += __shfl_xor_sync(0xffffffffu, rs[t][1], o);
+      }
+      if (g == 0) {
+        redl[warp * 16 + t * 8 + 2 * tig] = rs[t][0];
+        redl[warp * 16 + t * 8 + 2 * tig + 1] = rs[t][1];
+      }
     }
-    red[g * C::RED + warp * 4 + tig] = l0;
-    red[(g + 8) * C::RED + warp * 4 + tig] = l1;
     __syncthreads();   // P tiles and the row sums are complete
-    if (tid < 16) {
-      float lc = 0.f;
 #pragma unroll
-      for (int i = 0; i < 16; ++i) lc += red[tid * C::RED + i];
-      l_run[tid] = l_run[tid] * alpha[tid] + lc;
-    }
-    // ---- O = O * alpha + P V for this warp's HD/4 dimensions (DT tiles of 8), all 64 keys
-    {
-      const float a0 = alpha[g], a1 = alpha[g + 8];
+    for (int t = 0; t < QT; ++t)
 #pragma unroll
-      for (int nt = 0; nt < DT; ++nt) {
-        O[nt][0] *= a0;
-        O[nt][1] *= a0;
-        O[nt][2] *= a1;
-        O[nt][3] *= a1;
-        Ol[nt][0] *= a0;
-        Ol[nt][1] *= a0;
-        Ol[nt][2] *= a1;
-        Ol[nt][3] *= a1;
+      for (int i = 0; i < 2; ++i) {
+        const int j = t * 8 + 2 * tig + i;
+        lr[t][i] = lr[t][i] * al[t][i] + ((redl[j] + redl[16 + j]) + (redl[32 + j] + redl[48 + j]));
       }
-    }
+    // ---- O^T = O^T * alpha + V^T P^T: A = V^T (16 dims x 16 keys, transposed loads of the V
+    // tile), B = P^T (16 keys x 8 query rows), for this warp's dimensions and every query tile
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+      for (int t = 0; t < QT; ++t)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          O[mt][t][e] *= al[t][e & 1];
+          Ol[mt][t][e] *= al[t][e & 1];
+        }
     if (ok) {
 #pragma unroll
       for (int kk = 0; kk < ATT_UNIT / 16; ++kk) {
-        uint32_t ah[4], al[4];
-        const int prow = r8 + 8 * (mi & 1), pcol = kk * 16 + 8 * (mi >> 1);
-        ldsm_x4(smem_u32(Ph + prow * C::PSTRIDE + pcol * 2), ah[0], ah[1], ah[2], ah[3]);
-        ldsm_x4(smem_u32(Pl + prow * C::PSTRIDE + pcol * 2), al[0], al[1], al[2], al[3]);
+        uint32_t va[MT][4];
 #pragma unroll
-        for (int np = 0; np < DT / 2; ++np) {       // two dimension tiles per ldmatrix.x4.trans
-          const int key = kk * 16 + 8 * (mi & 1) + r8;
-          const int dim = db + 8 * (2 * np + (mi >> 1));
+        for (int mt = 0; mt < MT; ++mt) {
+          const int key = kk * 16 + r8 + 8 * (mi >> 1);
+          const int dim = db + 16 * mt + 8 * (mi & 1);
           const int hh = dim >> 6, cc = (dim & 63) >> 3;
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), b0, b1, b2, b3);
-          mma_bf16_16816(O[2 * np], ah[0], ah[1], ah[2], ah[3], b0, b1);
-          mma_bf16_16816(Ol[2 * np], al[0], al[1], al[2], al[3], b0, b1);
-          mma_bf16_16816(O[2 * np + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
-          mma_bf16_16816(Ol[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
+          ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), va[mt][0], va[mt][1],
+                    va[mt][2], va[mt][3]);
+        }
+#pragma unroll
+        for (int t = 0; t < QT; ++t) {
+          uint32_t ph0, ph1, pl0, pl1;   // P rows t*8 .. t*8+7, keys kk*16 ..: hi (0, 1), lo (2, 3)
+          const uint8_t* psrc = (mi >> 1) ? Pl : Ph;
+          ldsm_x4(smem_u32(psrc + (t * 8 + r8) * C::PSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), ph0, ph1, pl0, pl1);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) {
+            mma_bf16_16816(O[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], ph0, ph1);
+            mma_bf16_16816(Ol[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], pl0, pl1);
+          }
         }
       }
     }
@@ -390,22 +414,32 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
       const size_t pair = (size_t)h * ATT_SEG_MAX;
       const bool fits = nseg <= ATT_SEG_MAX;                   // always, for grids launch_attention makes
       if (!fits && tid == 0) set_error(p.err, ERR_CAPACITY);
-      if (tid < q && fits) {   // m_run[tid] and l_run[tid] were last written by this thread
-        float* ml = p.part_ml + ((size_t)(sl * q + tid) * H * ATT_SEG_MAX + pair + slot) * 2;
-        ml[0] = m_run[tid];
-        ml[1] = l_run[tid];
-      }
+      if (warp == 0 && g == 0 && fits) {   // the statistics of this thread's query rows
 #pragma unroll
-      for (int nt = 0; nt < DT; ++nt)
+        for (int t = 0; t < QT; ++t)
 #pragma unroll
-        for (int e = 0; e < 4; e += 2) {
-          const int j = g + 8 * (e >> 1);
-          if (j < q && fits) {
-            const int dim = db + 8 * nt + 2 * tig;
-            *reinterpret_cast<float2*>(p.part_o + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * HD + dim) =
-                make_float2(O[nt][e] + Ol[nt][e], O[nt][e + 1] + Ol[nt][e + 1]);
+          for (int i = 0; i < 2; ++i) {
+            const int j = t * 8 + 2 * tig + i;
+            if (j < q) {
+              float* ml = p.part_ml + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * 2;
+              ml[0] = mr[t][i];
+              ml[1] = lr[t][i];
+            }
           }
-        }
+      }
+      // O^T[mt][t][e] is dimension db + 16*mt + g + 8*(e >> 1) of query row t*8 + 2*tig + (e & 1)
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int t = 0; t < QT; ++t)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int j = t * 8 + 2 * tig + (e & 1);
+            if (j < q && fits) {
+              const int dim = db + 16 * mt + g + 8 * (e >> 1);
+              p.part_o[((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * HD + dim] = O[mt][t][e] + Ol[mt][t][e];
+            }
+          }
       if (p.trace.rec) t_part = globaltimer_ns();
       // the CTA's stores, then one release/acquire counter update by thread 0
       __syncthreads();
@@ -416,61 +450,79 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
       }
       __syncthreads();
       if (*s_last && fits) {
-        // ---- merge the pair's partials: w[j][s] = exp(m_s - max m), L_j = sum_s w[j][s] l_s
-        for (int t = tid; t < q * nseg; t += 128) {
-          const int j = t / nseg, s = t % nseg;
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(
-              p.part_ml + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + s) * 2));
-          ms[j * ATT_SEG_MAX + s] = v.x;
-          ls[j * ATT_SEG_MAX + s] = v.y;
-        }
-        __syncthreads();
-        if (tid < q) {
-          float mx = -INFINITY;
-          for (int s = 0; s < nseg; ++s) mx = fmaxf(mx, ms[tid * ATT_SEG_MAX + s]);
-          float L = 0.f;
-          for (int s = 0; s < nseg; ++s) {
-            const float m = ms[tid * ATT_SEG_MAX + s];
-            const float w = (m == -INFINITY) ? 0.f : expf(m - mx);
-            wg[tid * ATT_SEG_MAX + s] = w;
-            L += w * ls[tid * ATT_SEG_MAX + s];
-          }
-          inv[tid] = 1.0f / L;
-        }
-        __syncthreads();
-        // O_j = (sum_s w[j][s] o_s) / L_j: one (row, 4 dimensions) per thread, all partials in flight
-        for (int t = tid; t < q * D4; t += 128) {
-          const int j = t / D4, d4 = t % D4;
-          const float4* po =
-              reinterpret_cast<const float4*>(p.part_o + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair) * HD) + d4;
-          float4 v[ATT_SEG_MAX];
+        // ---- merge the pair's partials: w[j][s] = exp(m_s - max m), L_j = sum_s w[j][s] l_s,
+        // O_j = (sum_s w[j][s] o_s) / L_j.  Each thread takes (row, 4 dimensions) pairs, two
+        // per round; a round's partial outputs are requested together with the statistics
+        // (first round), so the merge costs one round trip per round.
+        constexpr int PR = 2;                           // pairs per thread per round
+        const int npairs = q * D4;
+        for (int base = 0; base < npairs; base += 128 * PR) {
+          float4 v[PR][ATT_SEG_MAX];
 #pragma unroll
-          for (int s = 0; s < ATT_SEG_MAX; ++s)
-            if (s < nseg) v[s] = __ldcg(po + (size_t)s * D4);
-          float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int pp = 0; pp < PR; ++pp) {
+            const int t = base + tid + 128 * pp;
+            if (t < npairs) {
+              const int j = t / D4, d4 = t % D4;
+              const float4* po =
+                  reinterpret_cast<const float4*>(p.part_o + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair) * HD) + d4;
 #pragma unroll
-          for (int s = 0; s < ATT_SEG_MAX; ++s) {
-            if (s < nseg) {
-              const float w = wg[j * ATT_SEG_MAX + s];
-              a.x += w * v[s].x;
-              a.y += w * v[s].y;
-              a.z += w * v[s].z;
-              a.w += w * v[s].w;
+              for (int s2 = 0; s2 < ATT_SEG_MAX; ++s2)
+                if (s2 < nseg) v[pp][s2] = __ldcg(po + (size_t)s2 * D4);
             }
           }
-          const float iv = inv[j];
-          const float4 o = make_float4(a.x * iv, a.y * iv, a.z * iv, a.w * iv);
-          const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + 4 * d4;
-          *reinterpret_cast<float4*>(p.out + idx) = o;
-          const __nv_bfloat16 h0 = __float2bfloat16_rn(o.x), h1 = __float2bfloat16_rn(o.y);
-          const __nv_bfloat16 h2 = __float2bfloat16_rn(o.z), h3 = __float2bfloat16_rn(o.w);
-          uint2 hi, lo;
-          hi.x = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-          hi.y = (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
-          lo.x = pack_bf16(o.x - __bfloat162float(h0), o.y - __bfloat162float(h1));
-          lo.y = pack_bf16(o.z - __bfloat162float(h2), o.w - __bfloat162float(h3));
-          *reinterpret_cast<uint2*>(p.out_hi + idx) = hi;
-          *reinterpret_cast<uint2*>(p.out_lo + idx) = lo;
+          if (base == 0) {
+            for (int t = tid; t < q * nseg; t += 128) {
+              const int j = t / nseg, s2 = t % nseg;
+              const float2 m2 = __ldcg(reinterpret_cast<const float2*>(
+                  p.part_ml + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + s2) * 2));
+              ms[j * ATT_SEG_MAX + s2] = m2.x;
+              ls[j * ATT_SEG_MAX + s2] = m2.y;
+            }
+            __syncthreads();
+            if (tid < q) {
+              float mx = -INFINITY;
+              for (int s2 = 0; s2 < nseg; ++s2) mx = fmaxf(mx, ms[tid * ATT_SEG_MAX + s2]);
+              float L = 0.f;
+              for (int s2 = 0; s2 < nseg; ++s2) {
+                const float m = ms[tid * ATT_SEG_MAX + s2];
+                const float w = (m == -INFINITY) ? 0.f : __expf(m - mx);
+                wg[tid * ATT_SEG_MAX + s2] = w;
+                L += w * ls[tid * ATT_SEG_MAX + s2];
+              }
+              inv[tid] = 1.0f / L;
+            }
+            __syncthreads();
+          }
+#pragma unroll
+          for (int pp = 0; pp < PR; ++pp) {
+            const int t = base + tid + 128 * pp;
+            if (t >= npairs) continue;
+            const int j = t / D4, d4 = t % D4;
+            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int s2 = 0; s2 < ATT_SEG_MAX; ++s2) {
+              if (s2 < nseg) {
+                const float w = wg[j * ATT_SEG_MAX + s2];
+                a.x += w * v[pp][s2].x;
+                a.y += w * v[pp][s2].y;
+                a.z += w * v[pp][s2].z;
+                a.w += w * v[pp][s2].w;
+              }
+            }
+            const float iv = inv[j];
+            const float4 o = make_float4(a.x * iv, a.y * iv, a.z * iv, a.w * iv);
+            const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + 4 * d4;
+            *reinterpret_cast<float4*>(p.out + idx) = o;
+            const __nv_bfloat16 h0 = __float2bfloat16_rn(o.x), h1 = __float2bfloat16_rn(o.y);
+            const __nv_bfloat16 h2 = __float2bfloat16_rn(o.z), h3 = __float2bfloat16_rn(o.w);
+            uint2 hi, lo;
+            hi.x = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+            hi.y = (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
+            lo.x = pack_bf16(o.x - __bfloat162float(h0), o.y - __bfloat162float(h1));
+            lo.y = pack_bf16(o.z - __bfloat162float(h2), o.w - __bfloat162float(h3));
+            *reinterpret_cast<uint2*>(p.out_hi + idx) = hi;
+            *reinterpret_cast<uint2*>(p.out_lo + idx) = lo;
+          }
         }
         if (tid == 0) p.counters[sl * H + h] = 0;
         ++merges;
@@ -499,11 +551,12 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
 size_t attention_smem_bytes(int hd) { return hd == 64 ? AttCfg<64>::SMEM : AttCfg<128>::SMEM; }
 
 cudaError_t attention_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(attention_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)AttCfg<64>::SMEM);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attention_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)AttCfg<128>::SMEM);
+  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(attention_kernel<64, 1>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(attention_kernel<64, 2>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(attention_kernel<128, 1>, a, (int)AttCfg<128>::SMEM)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attention_kernel<128, 2>, a, (int)AttCfg<128>::SMEM);
 }
 
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl) {
@@ -521,8 +574,9 @@ cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  if (p.hd == 64) return cudaLaunchKernelEx(&cfg, attention_kernel<64>, p);
-  return cudaLaunchKernelEx(&cfg, attention_kernel<128>, p);
+  const bool one = p.q <= 8;
+  if (p.hd == 64) return one ? cudaLaunchKernelEx(&cfg, attention_kernel<64, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<64, 2>, p);
+  return one ? cudaLaunchKernelEx(&cfg, attention_kernel<128, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<128, 2>, p);
 }
 
 }  // namespace sdsat
