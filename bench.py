@@ -144,7 +144,7 @@ def kv_bytes_per_layer_slot(shape):
 
 # ----------------------------------------------------------------------------- our arm
 class Runner:
-    def __init__(self, wl, device):
+    def __init__(self, wl, device, weights=None):
         import torch
         import synth
         import paper_2403_18647_gb300 as sd
@@ -157,7 +157,7 @@ class Runner:
         self.new = wl["new"]
         self.cap = self.P + 2 * self.new + 8 * self.q
         self.dev = device
-        self.weights = synth.make_model(self.shape, seed=0, device=device)
+        self.weights = weights if weights is not None else synth.make_model(self.shape, seed=0, device=device)
         torch.cuda.synchronize()
         self.ctx = sd.Context(self.shape, self.weights, max_position=self.cap + 64)
         self.kv = self.ctx.kv(self.b, self.cap)
@@ -285,6 +285,86 @@ class Runner:
                 self.step(1 if j % 2 == 0 else 2)
 
 
+def accept_rate(r, toks):
+    """Mean fraction of the k drafts accepted per verify step (draft step 2), from one
+    calibrated generation: a verify step emits 1 + m tokens per sequence."""
+    ver = [t for i, t in enumerate(toks) if i % 2 == 1]
+    if not ver:
+        return None
+    return round(statistics.mean((t / r.b - 1.0) / r.k for t in ver), 4)
+
+
+def step_latency(r, graphs, steps_per_gen, n):
+    """Per block step device latency (CUDA events around each replay): p10 / median / p90 in ms."""
+    torch = r.torch
+    if not graphs:
+        return None
+    r.reset()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    torch.cuda.synchronize()
+    ev[0].record()
+    for i in range(n):
+        j = i % steps_per_gen
+        if j == 0 and i > 0:
+            graphs[2].replay()
+        graphs[j % 2].replay()
+        ev[i + 1].record()
+    torch.cuda.synchronize()
+    t = sorted(ev[i].elapsed_time(ev[i + 1]) for i in range(n))
+    pick = lambda f: round(t[min(n - 1, int(f * n))], 4)
+    return {"p10": pick(0.1), "median": pick(0.5), "p90": pick(0.9), "steps": n}
+
+
+def run_plain(r, steps, warmup=3):
+    """The in-build baseline: plain decoding (q = 1, one token per forward) through the same
+    kernels, CUDA-graph replayed; tokens/s over `steps` forwards from the prompt."""
+    torch = r.torch
+    b, V, wl = r.b, r.shape.vocab, r.wl
+    steps = min(steps, r.new)
+    tok = torch.empty(b, dtype=torch.int32, device=r.dev)
+    lg = torch.empty(b, V, device=r.dev)
+    acc = torch.empty(b, dtype=torch.int32, device=r.dev)
+
+    def init():
+        r.ctx.kv_commit(r.kv, r.start_len, b)
+        tok.copy_(r.init_out.view(b, r.q)[:, 0])
+
+    def step():
+        r.ctx.block_forward(r.kv, tok, lg, b, 1)
+        if wl["temperature"] > 0:
+            r.ctx.accept_nucleus(r.kv, lg, tok, b, 1, 0, wl["top_p"], wl["temperature"], 1234, acc, tok,
+                                 top_k=wl["top_k"])
+        else:
+            r.ctx.accept_greedy(r.kv, lg, tok, b, 1, 0, acc, tok)
+
+    init()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for _ in range(warmup):
+            step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    init()
+    for _ in range(warmup):
+        g.replay()
+    init()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    init()
+    return {"tokens_per_s": round(b * steps / (ms / 1e3), 2), "ms_per_step": round(ms / steps, 4), "steps": steps,
+            "note": "plain greedy/nucleus decoding, q = 1, same kernels and graphs (in-build baseline)"}
+
+
 def run_ours(args, wl, rank, world):
     import torch
     import torch.distributed as dist
@@ -339,6 +419,9 @@ def run_ours(args, wl, rank, world):
     r.ctx.profile_begin(n_prof * (launches_per_step + 2) + 16)
     r.run_steps(n_prof, steps_per_gen, None)
     kstats = r.ctx.profile_end()
+    # --- per-step latency percentiles and the plain-decoding baseline on the same kernels
+    lat = step_latency(r, graphs, steps_per_gen, min(args.steps, 4 * steps_per_gen))
+    plain = run_plain(r, min(args.steps, 128))
     # --- e2e: the C ABI with host buffers (host builds inputs, reads outputs every step)
     e2e = run_e2e(r, args.steps, steps_per_gen)
     # --- bytes
@@ -372,6 +455,10 @@ def run_ours(args, wl, rank, world):
                    "l2": "inputs larger than L2 (%.1f GB of weights streamed per step)" % (Wb / 1e9),
                    "graphs": graphs is not None, "mma": "bf16 hi+lo activations x bf16 weights -> fp32"},
         "tokens_per_step": round(tokens / world / args.steps, 4),
+        "accept_rate": accept_rate(r, toks_cal),
+        "step_latency_ms": lat,
+        "plain_decoding": plain,
+        "speedup_vs_plain": round(value / world / plain["tokens_per_s"], 3) if plain else None,
         "expected_tokens_per_step": round(expected_tokens_per_step(r.k, wl["match"]), 4),
         "steps_per_generation": steps_per_gen,
         "step_hbm": {"bytes": int(step_bytes), "achieved_gbs": round(step_gbs, 1),
@@ -559,6 +646,44 @@ SWEEP_Q = [1, 2, 4, 6, 8, 11, 16]
 SWEEP_CTX = [512, 2048, 8192, 16384]
 
 
+def run_ksweep(args):
+    """k-sweep (one JSON line per k): block step time, tokens per step, accept rate and
+    tokens/s of the workload's generation loop for k adaptive tokens (q = k + 1), the same
+    weights throughout.  Checks that the step time stays almost flat in k (Sec. 3.4.1)."""
+    import torch
+    import synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    base = dict(WORKLOADS[args.config])
+    ks = [int(v) for v in args.ks.split(",")] if args.ks else list(range(1, 14))
+    weights = synth.make_model(synth.SHAPES[base["shape"]], seed=0, device=dev)
+    for k in ks:
+        wl = dict(base, k=k)
+        r = Runner(wl, dev, weights=weights)
+        steps_per_gen, lens, toks_cal, flags = r.calibrate()
+        graphs = r.capture()
+        r.reset()
+        r.run_steps(4, steps_per_gen, graphs)
+        r.reset()
+        n = steps_per_gen
+        em0 = r.ctx.kv_emitted(r.kv).sum().item()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        r.run_steps(n, steps_per_gen, graphs)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        tokens = r.ctx.kv_emitted(r.kv).sum().item() - em0
+        print(json.dumps({"kind": "ksweep", "workload": args.config, "k": k, "q": k + 1, "steps": n,
+                          "ms_per_step": round(ms / n, 4), "tokens_per_step": round(tokens / r.b / n, 4),
+                          "expected_tokens_per_step": round(expected_tokens_per_step(k, wl["match"]), 4),
+                          "accept_rate": accept_rate(r, toks_cal), "tokens_per_s": round(tokens / (ms / 1e3), 2),
+                          "device_error_flags": flags | r.ctx.get_error()}), flush=True)
+        del graphs, r
+        torch.cuda.synchronize()
+
+
 def run_sweep(args):
     """Kernel sweeps on 7B shapes (one JSON line per case): the skinny GEMM with M = q against
     bf16 weights, and block-causal attention of q rows (32 heads x 128) against a bf16 cache.
@@ -643,9 +768,14 @@ def main():
     ap.add_argument("--m", type=int, default=0, help="sweep one M (GEMM) or q (attention)")
     ap.add_argument("--ctx", type=int, default=0, help="sweep one attention context length")
     ap.add_argument("--reps", type=int, default=50)
+    ap.add_argument("--ksweep", action="store_true", help="k-sweep of the generation loop (k = 1..13)")
+    ap.add_argument("--ks", default="", help="k values for --ksweep, comma separated")
     args = ap.parse_args()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.ksweep:
+        run_ksweep(args)
         return
     if args.warmup < 3:
         args.warmup = 3

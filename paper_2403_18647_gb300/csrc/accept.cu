@@ -122,8 +122,7 @@ __device__ int row_argmax(const float* row, int V, uint32_t* err, float* redf, i
   float best = -INFINITY;
   int bi = 0x7FFFFFFF;
   bool nan = false;
-  for (int i = threadIdx.x; i < V; i += blockDim.x) {
-    float x = __ldcg(row + i);
+  auto take = [&](float x, int i) {
     if (x != x) {
       nan = true;
       x = -INFINITY;
@@ -132,7 +131,31 @@ __device__ int row_argmax(const float* row, int V, uint32_t* err, float* redf, i
       best = x;
       bi = i;
     }
+  };
+  // float4 loads, a round of RN per thread issued before any is compared (the row is one
+  // L2 round trip per round, not one per element); a thread visits its ids in increasing order
+  constexpr int RN = 8;
+  const bool vec = (reinterpret_cast<uintptr_t>(row) & 15u) == 0;
+  const int V4 = vec ? V / 4 : 0;
+  for (int i0 = 0; i0 < V4; i0 += RN * (int)blockDim.x) {
+    float4 v[RN];
+#pragma unroll
+    for (int u = 0; u < RN; ++u) {
+      const int i = i0 + u * (int)blockDim.x + threadIdx.x;
+      if (i < V4) v[u] = __ldcg(reinterpret_cast<const float4*>(row) + i);
+    }
+#pragma unroll
+    for (int u = 0; u < RN; ++u) {
+      const int i = i0 + u * (int)blockDim.x + threadIdx.x;
+      if (i < V4) {
+        take(v[u].x, 4 * i);
+        take(v[u].y, 4 * i + 1);
+        take(v[u].z, 4 * i + 2);
+        take(v[u].w, 4 * i + 3);
+      }
+    }
   }
+  for (int i = 4 * V4 + threadIdx.x; i < V; i += blockDim.x) take(__ldcg(row + i), i);
   if (nan) set_error(err, ERR_NAN_LOGITS);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
