@@ -96,6 +96,27 @@ def attend(q: np.ndarray, K: np.ndarray, V: np.ndarray, n_visible: Sequence[int]
     return out
 
 
+def attend_rows(q: np.ndarray, K: np.ndarray, V: np.ndarray, L0: int,
+                visible: Sequence[Sequence[int]]) -> np.ndarray:
+    """softmax(q k^T / sqrt(hd)) v per row and head over the committed slots [0, L0) and the
+    block slots L0 + i for i in visible[j] (ascending), the tree-attention mask of Sec. 2.1.2.
+
+    With visible[j] = 0..j this is attend() with n_visible[j] = L0 + j + 1, in the same
+    slot order, so the two agree bit for bit.
+    """
+    n, H, hd = q.shape
+    out = np.empty_like(q)
+    scale = 1.0 / math.sqrt(hd)
+    for j in range(n):
+        slots = list(range(L0)) + [L0 + int(i) for i in sorted(visible[j])]
+        for h in range(H):
+            s = (K[h, slots] @ q[j, h]) * scale
+            e = np.exp(s - s.max())
+            p = e / e.sum()
+            out[j, h] = p @ V[h, slots]
+    return out
+
+
 class Weights:
     """fp64 view of a synth-style weight dict, widened lazily (optionally cached)."""
 
@@ -144,13 +165,16 @@ class KVCache:
 def block_forward(W: Weights, kv: KVCache, seq: int, tokens: Sequence[int],
                   positions: Optional[Sequence[int]] = None,
                   layers: Optional[Sequence[int]] = None,
-                  final: bool = True) -> np.ndarray:
+                  final: bool = True,
+                  visible: Optional[Sequence[Sequence[int]]] = None) -> np.ndarray:
     """Logits [n, V] of the n = q block rows of sequence `seq`.
 
     Block rows occupy cache slots len .. len+n-1 (written here; `kv.len` is
     not advanced -- committing is the acceptance step's job).  RoPE uses
     `positions` when given, else the slot index.  `layers` restricts the
-    pass to a subset (used only to time a bounded sample).
+    pass to a subset (used only to time a bounded sample).  `visible[j]`,
+    when given, lists the block rows row j attends to (a tree mask, see
+    oracle/tree.py); the default is block-causal (rows 0..j).
     """
     shape = W.shape
     n = len(tokens)
@@ -171,7 +195,10 @@ def block_forward(W: Weights, kv: KVCache, seq: int, tokens: Sequence[int],
         k = rope(k, pos, shape.rope_theta)
         kv.K[l][seq][:, L0:L0 + n] = k.transpose(1, 0, 2)
         kv.V[l][seq][:, L0:L0 + n] = v.transpose(1, 0, 2)
-        o = attend(q, kv.K[l][seq], kv.V[l][seq], n_visible)
+        if visible is None:
+            o = attend(q, kv.K[l][seq], kv.V[l][seq], n_visible)
+        else:
+            o = attend_rows(q, kv.K[l][seq], kv.V[l][seq], L0, visible)
         h = h + linear(o.reshape(n, H * hd), W.get("wo", l))
         x = rmsnorm(h, W.get("ffn_norm", l), eps)
         a = silu(linear(x, W.get("w_gate", l))) * linear(x, W.get("w_up", l))
