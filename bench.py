@@ -44,6 +44,10 @@ WORKLOADS = {
     # 7B shape, nucleus verification (top_p 0.95, T 0.2), batch 4, prompts of 1024
     "7b-nucleus": dict(shape="7b", batch=4, prompt=1024, new=256, k=5, temperature=0.2, top_p=0.95, top_k=0,
                        match=0.6),
+    # 7B shape, tree draft step 2 (Sec. 2.1.2): nucleus T 0.2, top_p 0.95, top_k 10 (the paper's
+    # nucleus setting), k = 5 = tree depth, two chains of drafts below the root (q = 11)
+    "7b-tree": dict(shape="7b", batch=1, prompt=2048, new=256, k=5, temperature=0.2, top_p=0.95, top_k=10,
+                    match=0.6, width=2, match2=0.4),
     # tiny correctness shape
     "tiny": dict(shape="tiny", batch=1, prompt=128, new=64, k=5, temperature=0.0, top_p=1.0, top_k=0, match=0.7),
 }
@@ -57,9 +61,29 @@ GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 lau
                        "algorithmic), ratio scaled to the average launch; bytes per launch")
 
 
-def expected_tokens_per_step(k: int, match: float) -> float:
-    """Two steps emit 2 + m tokens, m = leading matches of k drafts (Sec. 2.1.1)."""
-    return (2.0 + sum(match ** j for j in range(1, k + 1))) / 2.0
+def expected_tokens_per_step(k: int, match: float, matches=None) -> float:
+    """Two steps emit 2 + m tokens, m = leading matches of k drafts (Sec. 2.1.1); with several
+    branches of independent stub coins (match rates `matches`), m is the longest accepted branch:
+    P(m >= i) = 1 - prod_w (1 - p_w^i)."""
+    ps = list(matches) if matches else [match]
+    tail = 0.0
+    for i in range(1, k + 1):
+        miss = 1.0
+        for p in ps:
+            miss *= 1.0 - p ** i
+        tail += 1.0 - miss
+    return (2.0 + tail) / 2.0
+
+
+def branch_matches(wl):
+    """Stub match rate of every branch of the workload's draft tree (one branch: the chain)."""
+    w = wl.get("width", 1)
+    return [wl["match"]] + [wl.get("match2", wl["match"])] * (w - 1)
+
+
+def chains_parent(width: int, k: int):
+    """Parent rows of the draft tree of `width` chains of k drafts below the root (row 0)."""
+    return [-1] + [0 if i == 0 else 1 + w * k + i - 1 for w in range(width) for i in range(k)]
 
 
 def peaks():
@@ -152,26 +176,33 @@ class Runner:
         self.wl = wl
         self.shape = synth.SHAPES[wl["shape"]]
         self.b, self.k = wl["batch"], wl["k"]
-        self.q = self.k + 1
+        self.q = self.k + 1                       # draft step 1 block rows
+        self.width = wl.get("width", 1)
+        self.tree = self.width > 1
+        self.q2 = 1 + self.width * self.k         # draft step 2 block rows (the tree; the chain: q)
+        self.qmax = max(self.q, self.q2)
         self.P = wl["prompt"]
         self.new = wl["new"]
-        self.cap = self.P + 2 * self.new + 8 * self.q
+        self.cap = self.P + 2 * self.new + 8 * self.qmax
         self.dev = device
         self.weights = weights if weights is not None else synth.make_model(self.shape, seed=0, device=device)
         torch.cuda.synchronize()
         self.ctx = sd.Context(self.shape, self.weights, max_position=self.cap + 64)
         self.kv = self.ctx.kv(self.b, self.cap)
         V = self.shape.vocab
-        self.logits = torch.empty(self.b * self.q, V, device=device)
-        self.toks = torch.zeros(self.b * self.q, dtype=torch.int32, device=device)
+        self.logits = torch.empty(self.b * self.qmax, V, device=device)
+        self.toks = torch.zeros(self.b * self.qmax, dtype=torch.int32, device=device)
         self.acc = torch.ones(self.b, dtype=torch.int32, device=device)
-        self.out = torch.zeros(self.b * self.q, dtype=torch.int32, device=device)
+        self.out = torch.zeros(self.b * self.qmax, dtype=torch.int32, device=device)
+        self.parent = torch.tensor(chains_parent(self.width, self.k) * self.b, dtype=torch.int32, device=device)
         self.prompts = [synth.prompt_ids(0, s, self.P, self.shape.adaptive_id, device) for s in range(self.b)]
         for s in range(self.b):
             self.ctx.prefill(self.kv, s, self.prompts[s][:-1].contiguous())
+        self.first = torch.stack([p[-1] for p in self.prompts]).to(torch.int32)
+        # the loop starts as if a draft step 2 block (q2 rows) had just emitted the last prompt token
         self.init_out = torch.zeros_like(self.out)
         for s in range(self.b):
-            self.init_out[s * self.q] = self.prompts[s][-1]
+            self.init_out[s * self.q2] = self.prompts[s][-1]
         self.init_acc = torch.ones_like(self.acc)
         self.start_len = torch.full((self.b,), self.P - 1, dtype=torch.int32, device=device)
         self._make_table()
@@ -194,7 +225,7 @@ class Runner:
         n_ref = 2 * self.new + 8 * self.q
         ref = torch.zeros(n_ref, self.b, dtype=torch.int32, device=self.dev)
         lg = torch.empty(self.b, self.shape.vocab, device=self.dev)
-        tok = self.init_out.view(self.b, self.q)[:, 0].clone()   # a copy: init_out must stay intact
+        tok = self.first.clone()
         acc = torch.empty(self.b, dtype=torch.int32, device=self.dev)
         wl = self.wl
         n_run = min(n_ref, self.cap - self.P)
@@ -208,11 +239,13 @@ class Runner:
             ref[i] = tok
         self.ctx.kv_commit(self.kv, self.start_len, self.b)
         self.stride = self.cap + 32
-        table = torch.zeros(self.b, self.stride, dtype=torch.int32, device=self.dev)
-        for s in range(self.b):
-            full = torch.zeros(self.stride, dtype=torch.int32, device=self.dev)
-            full[self.P:self.P + n_run] = ref[:n_run, s]
-            table[s] = self.synth.stub_table(0, s, full, wl["match"], self.shape.vocab)
+        # [width][b][stride]: branch w's stub (own coins) with its match rate
+        table = torch.zeros(self.width, self.b, self.stride, dtype=torch.int32, device=self.dev)
+        for w, match in enumerate(branch_matches(wl)):
+            for s in range(self.b):
+                full = torch.zeros(self.stride, dtype=torch.int32, device=self.dev)
+                full[self.P:self.P + n_run] = ref[:n_run, s]
+                table[w, s] = self.synth.stub_table(w, s, full, match, self.shape.vocab)
         self.table = table.contiguous()
         self.ref = ref
 
@@ -222,10 +255,27 @@ class Runner:
         self.acc.copy_(self.init_acc)
 
     def step(self, mode):
-        self.ctx.build_block(self.kv, mode, self.out, self.acc, self.toks, self.b, self.q,
-                             draft_table=self.table if mode == 2 else None, table_stride=self.stride)
-        self.ctx.block_forward(self.kv, self.toks, self.logits, self.b, self.q)
-        self.accept(0 if mode == 1 else self.k)
+        if not self.tree:
+            self.ctx.build_block(self.kv, mode, self.out, self.acc, self.toks, self.b, self.q,
+                                 draft_table=self.table if mode == 2 else None, table_stride=self.stride)
+            self.ctx.block_forward(self.kv, self.toks, self.logits, self.b, self.q)
+            self.accept(0 if mode == 1 else self.k)
+        elif mode == 1:
+            self.ctx.build_tree_block(self.kv, 1, self.out, self.q2, self.acc, self.toks, self.b, self.k)
+            self.ctx.block_forward(self.kv, self.toks, self.logits, self.b, self.q)
+            self.accept(0)
+        else:
+            self.ctx.build_tree_block(self.kv, 2, self.out, self.q, self.acc, self.toks, self.b, self.k,
+                                      draft_tables=self.table, width=self.width, table_stride=self.stride)
+            self.forward_accept_tree()
+
+    def forward_accept_tree(self):
+        """Draft step 2 as a tree (Sec. 2.1.2): tree forward, then tree verification, compaction
+        of the accepted branch's KV rows and commit."""
+        wl = self.wl
+        self.ctx.block_forward_tree(self.kv, self.toks, self.parent, self.logits, self.b, self.q2)
+        self.ctx.accept_tree(self.kv, self.logits, self.toks, self.parent, self.b, self.q2, self.acc, self.out,
+                             temperature=wl["temperature"], top_p=wl["top_p"], seed=1234, top_k=wl["top_k"])
 
     def calibrate(self):
         """One generation with host checks: the number of steps it takes and the tokens
@@ -327,7 +377,7 @@ def run_plain(r, steps, warmup=3):
 
     def init():
         r.ctx.kv_commit(r.kv, r.start_len, b)
-        tok.copy_(r.init_out.view(b, r.q)[:, 0])
+        tok.copy_(r.first)
 
     def step():
         r.ctx.block_forward(r.kv, tok, lg, b, 1)
@@ -424,9 +474,10 @@ def run_ours(args, wl, rank, world):
     plain = run_plain(r, min(args.steps, 128))
     # --- e2e: the C ABI with host buffers (host builds inputs, reads outputs every step)
     e2e = run_e2e(r, args.steps, steps_per_gen)
-    # --- bytes
-    M = r.b * r.q
-    gb = gemm_bytes(shape, M)
+    # --- bytes (steps alternate q-row and q2-row blocks; for the chain q2 = q)
+    rows = [r.q if i % 2 == 0 else r.q2 for i in range(len(lens))]
+    gb1, gb2 = gemm_bytes(shape, r.b * r.q), gemm_bytes(shape, r.b * r.q2)
+    gb = {n: (gb1[n] + gb2[n]) / 2.0 for n in gb1}
     g_bytes = sum(gb[n] * kstats.get(n, (0, 0))[0] for n in gb)
     g_ms = sum(kstats.get(n, (0, 0.0))[1] for n in gb)
     g_launches = sum(kstats.get(n, (0, 0))[0] for n in gb)
@@ -435,22 +486,25 @@ def run_ours(args, wl, rank, world):
     # per-step algorithmic bytes over one calibrated generation
     Wb = weight_bytes(shape)
     slot = kv_bytes_per_layer_slot(shape) * shape.n_layers
-    kv_read = [sum(l + r.q for l in ln) * slot for ln in lens]
-    kv_write = M * slot
-    logit_b = M * shape.vocab * 4
-    step_bytes = Wb + statistics.mean(kv_read) + kv_write + logit_b
+    kv_read = [sum(l + q for l in ln) * slot for ln, q in zip(lens, rows)]
+    kv_write = [r.b * q * slot for q in rows]
+    logit_b = [r.b * q * shape.vocab * 4 for q in rows]
+    step_bytes = Wb + statistics.mean(kv_read) + statistics.mean(kv_write) + statistics.mean(logit_b)
     ms_step = ms / args.steps
     step_gbs = step_bytes / (ms_step / 1e3) / 1e9
-    # --- gpu launches in the timed region: our kernels only
+    # --- gpu launches in the timed region: our kernels only (a tree step adds its prep and
+    # compaction kernels)
     resets = sum(1 for i in range(args.steps) if i % steps_per_gen == 0 and i > 0)
-    gpu_launches = args.steps * launches_per_step + resets
+    tree_steps = sum(1 for i in range(args.steps) if (i % steps_per_gen) % 2 == 1) if r.tree else 0
+    gpu_launches = args.steps * launches_per_step + 2 * tree_steps + resets
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed 0)",
                    "global_batch": r.b * world, "seq_len": r.P, "new_tokens": r.new, "k": r.k, "q": r.q,
-                   "draft_stub_match": wl["match"], "temperature": wl["temperature"], "top_p": wl["top_p"],
+                   "draft_stub_match": branch_matches(wl) if r.tree else wl["match"],
+                   "temperature": wl["temperature"], "top_p": wl["top_p"], "top_k": wl["top_k"],
                    "parallelism": "replicas%d" % world if world > 1 else "single",
                    "l2": "inputs larger than L2 (%.1f GB of weights streamed per step)" % (Wb / 1e9),
                    "graphs": graphs is not None, "mma": "bf16 hi+lo activations x bf16 weights -> fp32"},
@@ -459,7 +513,7 @@ def run_ours(args, wl, rank, world):
         "step_latency_ms": lat,
         "plain_decoding": plain,
         "speedup_vs_plain": round(value / world / plain["tokens_per_s"], 3) if plain else None,
-        "expected_tokens_per_step": round(expected_tokens_per_step(r.k, wl["match"]), 4),
+        "expected_tokens_per_step": round(expected_tokens_per_step(r.k, wl["match"], branch_matches(wl)), 4),
         "steps_per_generation": steps_per_gen,
         "step_hbm": {"bytes": int(step_bytes), "achieved_gbs": round(step_gbs, 1),
                      "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4),
@@ -475,6 +529,9 @@ def run_ours(args, wl, rank, world):
                     for k, v in kstats.items()},
         "e2e": e2e, "gpu_launches": gpu_launches, "device_error_flags": flags,
     }
+    if r.tree:
+        out["config"].update({"tree_width": r.width, "q2": r.q2,
+                              "tree": "width chains of k drafts below the root (Sec. 2.1.2)"})
     if clk:
         out["clocks"] = clk
     return r, out
@@ -483,42 +540,49 @@ def run_ours(args, wl, rank, world):
 def run_e2e(r, steps, steps_per_gen):
     """The decode loop a host program writes against the C ABI: every step the host builds
     the block input from the previous step's emitted tokens (pinned buffer -> device copy),
-    calls block_forward and accept, copies the emitted tokens and accepted lengths back and
-    reads them before the next step."""
+    calls block_forward and accept (a tree step: the tree forward and tree accept), copies the
+    emitted tokens and accepted lengths back and reads them before the next step."""
     import torch
-    b, q, k = r.b, r.q, r.k
-    tok_h = torch.zeros(b * q, dtype=torch.int32).pin_memory()
-    out_h = torch.zeros(b * q, dtype=torch.int32).pin_memory()
+    b, k = r.b, r.k
+    qm = r.qmax
+    tok_h = torch.zeros(b * qm, dtype=torch.int32).pin_memory()
+    out_h = torch.zeros(b * qm, dtype=torch.int32).pin_memory()
     acc_h = torch.zeros(b, dtype=torch.int32).pin_memory()
     table = r.table.cpu()
     adaptive = [r.shape.adaptive_id] * k
     r.reset()
     torch.cuda.synchronize()
-    lens = [r.P - 1] * b
-    last_out = [[int(r.prompts[s][-1])] + [0] * k for s in range(b)]
-    last_acc = [1] * b
+
+    def start():
+        return [r.P - 1] * b, [[int(r.prompts[s][-1])] for s in range(b)], [1] * b
+
+    lens, last_out, last_acc = start()
     tokens = 0
+    h2d = d2h = 0
     st = torch.cuda.current_stream()
     t0 = time.perf_counter()
     for i in range(steps):
         j = i % steps_per_gen
         if j == 0 and i > 0:
             r.reset()
-            lens = [r.P - 1] * b
-            last_out = [[int(r.prompts[s][-1])] + [0] * k for s in range(b)]
-            last_acc = [1] * b
+            lens, last_out, last_acc = start()
         mode = 1 if j % 2 == 0 else 2
+        q = r.q if mode == 1 else r.q2
         blk = []
         for s in range(b):
             if mode == 1:
                 blk += [last_out[s][last_acc[s] - 1]] + adaptive
             else:
-                blk += [last_out[s][0]] + [int(table[s, lens[s] + jj]) for jj in range(1, q)]
-        tok_h.copy_(torch.tensor(blk, dtype=torch.int32))
-        r.toks.copy_(tok_h, non_blocking=True)
-        r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
-        r.accept(0 if mode == 1 else k)
-        out_h.copy_(r.out, non_blocking=True)
+                blk += [last_out[s][0]] + [int(table[w, s, lens[s] + jj]) for w in range(r.width)
+                                           for jj in range(1, k + 1)]
+        tok_h[:b * q].copy_(torch.tensor(blk, dtype=torch.int32))
+        r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
+        if mode == 2 and r.tree:
+            r.forward_accept_tree()
+        else:
+            r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
+            r.accept(0 if mode == 1 else k)
+        out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
         acc_h.copy_(r.acc, non_blocking=True)
         st.synchronize()
         o = out_h.tolist()
@@ -528,9 +592,11 @@ def run_e2e(r, steps, steps_per_gen):
             last_acc[s] = a[s]
             lens[s] += a[s]
         tokens += sum(a)
+        h2d += b * q * 4
+        d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
-    return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": b * q * 4,
-            "d2h_bytes_per_step": b * q * 4 + b * 4, "launch": "eager C-ABI calls, host sync each step"}
+    return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d / steps, 1),
+            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": "eager C-ABI calls, host sync each step"}
 
 
 # ----------------------------------------------------------------------------- CPU oracle
@@ -544,7 +610,7 @@ def oracle_sample(shape_name, wl, weights_gpu=None, n_layers=2, repeat=1, gen_de
     import synth
     from oracle import model as OM
     shape = synth.SHAPES[shape_name]
-    q = wl["k"] + 1
+    q = mean_rows(wl)
     P = wl["prompt"]
 
     def provider(name, layer):
@@ -580,15 +646,20 @@ def oracle_sample(shape_name, wl, weights_gpu=None, n_layers=2, repeat=1, gen_de
     return shape.n_layers * per_layer + t_head, {"per_layer_s": per_layer, "head_s": t_head}
 
 
+def mean_rows(wl):
+    """Block rows of the workload's average step (steps alternate k + 1 and 1 + width * k rows)."""
+    return round((wl["k"] + 1 + 1 + wl.get("width", 1) * wl["k"]) / 2)
+
+
 def cpu_baseline(args, wl, weights_gpu):
-    tps = expected_tokens_per_step(wl["k"], wl["match"])
+    tps = expected_tokens_per_step(wl["k"], wl["match"], branch_matches(wl))
     dev = next(iter(weights_gpu["layers"][0].values())).device if weights_gpu is not None else "cpu"
     t_step, det = oracle_sample(wl["shape"], wl, weights_gpu, n_layers=2, gen_device=dev)
     return {"value": round(tps / t_step, 4), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
             "sample": ("one q=%d block step at context %d: 2 of %d decoder layers timed (weights widened and cached "
                        "first) plus the final norm + LM head, extrapolated to all layers (%.2f s/layer, %.2f s head); "
                        "tokens/step = %.3f, the stub's expectation" %
-                       (wl["k"] + 1, wl["prompt"], __import__("synth").SHAPES[wl["shape"]].n_layers,
+                       (mean_rows(wl), wl["prompt"], __import__("synth").SHAPES[wl["shape"]].n_layers,
                         det["per_layer_s"], det["head_s"], tps)),
             "s_per_step": round(t_step, 3)}
 
@@ -599,8 +670,8 @@ def run_reference(args, wl, rank, world):
     import synth
     from oracle import model as OM
     shape = synth.SHAPES[wl["shape"]]
-    tps = expected_tokens_per_step(wl["k"], wl["match"])
-    q = wl["k"] + 1
+    tps = expected_tokens_per_step(wl["k"], wl["match"], branch_matches(wl))
+    q = mean_rows(wl)
     P = wl["prompt"]
     W = OM.Weights(shape, provider=lambda n, l: synth.make_weight(shape, n, l, 0, "cpu"), cache=True)
     small = synth.ModelShape("sample", 1, shape.d_model, shape.n_heads, shape.head_dim, shape.ffn_dim,
@@ -675,9 +746,9 @@ def run_ksweep(args):
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1)
         tokens = r.ctx.kv_emitted(r.kv).sum().item() - em0
-        print(json.dumps({"kind": "ksweep", "workload": args.config, "k": k, "q": k + 1, "steps": n,
+        print(json.dumps({"kind": "ksweep", "workload": args.config, "k": k, "q": k + 1, "q2": r.q2, "steps": n,
                           "ms_per_step": round(ms / n, 4), "tokens_per_step": round(tokens / r.b / n, 4),
-                          "expected_tokens_per_step": round(expected_tokens_per_step(k, wl["match"]), 4),
+                          "expected_tokens_per_step": round(expected_tokens_per_step(k, wl["match"], branch_matches(wl)), 4),
                           "accept_rate": accept_rate(r, toks_cal), "tokens_per_s": round(tokens / (ms / 1e3), 2),
                           "device_error_flags": flags | r.ctx.get_error()}), flush=True)
         del graphs, r

@@ -62,6 +62,7 @@ typedef enum {
 #define SDSAT_DEV_CAPACITY 0x4u    /* a block row fell past the KV capacity; not written */
 #define SDSAT_DEV_TOKEN 0x8u       /* a token id outside [0, vocab); id 0 used instead */
 #define SDSAT_DEV_POSITION 0x10u   /* a RoPE position outside [0, max_position); clamped */
+#define SDSAT_DEV_TREE 0x20u       /* a tree parent that is not an earlier row; read as the root */
 
 #define SDSAT_MAX_Q 16           /* block rows per sequence (k <= 15 adaptive tokens) */
 #define SDSAT_MAX_ROWS 64        /* batch * q rows per block forward */
@@ -224,6 +225,67 @@ SDSAT_API sdsat_status sdsat_kv_emitted(sdsat_ctx* ctx, sdsat_kv* kv, int64_t* e
 SDSAT_API sdsat_status sdsat_build_block(sdsat_ctx* ctx, sdsat_kv* kv, int mode, const int32_t* prev_out_dev,
                                const int32_t* prev_acc_dev, const int32_t* draft_table_dev,
                                int table_stride, int b, int q, int32_t* tokens_out_dev);
+
+/* ---- tree-structured draft step 2 (Sec. 2.1.2) ----------------------------------- */
+/* A tree block holds q rows per sequence: the nodes of a draft tree in
+ * topological order.  parent_dev int32 [b*q]: entry s*q + j is the parent row of
+ * row j of sequence s; row 0 is the root (parent -1, the token y_{n+1} of draft
+ * step 1) and every other row's parent is an earlier row (parent[j] < j).
+ * Anything else sets device bit TREE and the row is read as a child of the root.
+ * Row j has depth(j) = number of edges to the root, occupies KV slot len[s] + j
+ * and sits at position len[s] + depth(j).  A chain (parent[j] = j - 1) is the
+ * ordinary block of sdsat_block_forward / sdsat_accept_*. */
+
+/* Tree block forward: as sdsat_block_forward, with RoPE positions
+ * len[s] + depth(j) and the tree attention mask -- row j attends to the committed
+ * slots [0, len[s]) and to the slots of its ancestors and itself only.
+ * tokens_dev int32 [b*q]; logits_dev fp32 [b*q][vocab], written.  len is not
+ * advanced.  Errors: EINVAL (null pointer, b < 1, b > kv batch, q < 1,
+ * q > SDSAT_MAX_Q, b*q > SDSAT_MAX_ROWS); device bits TREE, CAPACITY. */
+SDSAT_API sdsat_status sdsat_block_forward_tree(sdsat_ctx* ctx, sdsat_kv* kv, const int32_t* tokens_dev,
+                                                const int32_t* parent_dev, int b, int q, float* logits_dev);
+
+/* Tree verification and commit (Sec. 2.1.2: the longest branch of the tree that
+ * is verified and accepted is the loop's result).
+ *   targets  t_j = the selection of sdsat_accept_nucleus (temperature > 0) or
+ *            argmax (temperature == 0) of row j's logits, the produced token at
+ *            position len[s] + depth(j) + 1;
+ *   accepted row 0 always; row j > 0 iff its parent p is accepted and
+ *            tokens[s*q + j] == t_p (the chain test of Eq. 3 along each branch);
+ *   path     n_0 = 0, n_1, ..., n_m: the root path of the deepest accepted row
+ *            (the lowest row index among equally deep ones).
+ * out_tokens_dev   int32 [b*q]: t_{n_0} .. t_{n_m}, then -1.
+ * accepted_len_dev int32 [b]: 1 + m.
+ * path_dev         int32 [b*q]: n_0 .. n_m, then -1; may be NULL.
+ * The K and V rows of the path always move to slots len[s] + 1 .. len[s] + m
+ * (slot len[s] + i receives row n_i's rows, which were rotated at position
+ * len[s] + i already), so the cache holds the accepted branch contiguously;
+ * commit != 0 then advances len[s] by 1 + m (with commit == 0, an explicit
+ * sdsat_kv_commit of len[s] + 1 + m commits it later).
+ * Other arguments as sdsat_accept_nucleus.  Errors: EINVAL (null parent_dev,
+ * temperature < 0 or NaN, the sdsat_accept_nucleus conditions), EUNSUPPORTED
+ * (temperature > 0 and vocab > 32768); device bit TREE. */
+SDSAT_API sdsat_status sdsat_accept_tree(sdsat_ctx* ctx, sdsat_kv* kv, const float* logits_dev,
+                                         const int32_t* tokens_dev, const int32_t* parent_dev, int b, int q,
+                                         float temperature, float top_p, uint64_t rng_seed, int top_k,
+                                         int32_t* accepted_len_dev, int32_t* out_tokens_dev, int32_t* path_dev,
+                                         int commit);
+
+/* Block building for tree loops, where consecutive blocks differ in size:
+ *   mode 1 (draft step 1): q = k + 1 rows; row 0 = prev_out[s*prev_q + prev_acc[s] - 1],
+ *     rows 1..k = the adaptive ids;
+ *   mode 2 (draft step 2): the tree of `width` chains of k drafts below the root,
+ *     q = 1 + width*k rows (parent of row 1 + w*k is 0, of row 1 + w*k + i is
+ *     row w*k + i); row 0 = prev_out[s*prev_q]; row 1 + w*k + i - 1 (1 <= i <= k)
+ *     = draft_tables_dev[(w*B + s)*table_stride + len[s] + i] with B the KV batch
+ *     (branch w's draft for position len[s] + i).  Without tables (width 1 only)
+ *     row i = prev_out[s*prev_q + i] (k < prev_q).
+ * tokens_out_dev int32 [b*q].  Errors: EINVAL (q > SDSAT_MAX_Q, b*q > SDSAT_MAX_ROWS,
+ * table_stride < max_len + SDSAT_MAX_Q, the sdsat_build_block conditions). */
+SDSAT_API sdsat_status sdsat_build_tree_block(sdsat_ctx* ctx, sdsat_kv* kv, int mode, const int32_t* prev_out_dev,
+                                              int prev_q, const int32_t* prev_acc_dev,
+                                              const int32_t* draft_tables_dev, int width, int table_stride, int b,
+                                              int k, int32_t* tokens_out_dev);
 
 /* Run n prompt tokens of sequence `seq` through the model in blocks of up to
  * SDSAT_MAX_Q rows and commit them (len[seq] += n).  No logits are produced.

@@ -88,6 +88,9 @@ def _lib():
             "sdsat_trace_end": [P, P, I, ctypes.POINTER(I)],
             "sdsat_profile_end": [P, ctypes.POINTER(KernelStat), I, ctypes.POINTER(I)],
             "sdsat_build_block": [P, P, I, P, P, P, I, I, I, P],
+            "sdsat_block_forward_tree": [P, P, P, P, I, I, P],
+            "sdsat_accept_tree": [P, P, P, P, P, I, I, F, F, U64, I, P, P, P, I],
+            "sdsat_build_tree_block": [P, P, I, P, I, P, P, I, I, I, I, P],
             "sdsat_prefill": [P, P, I, P, I],
             "sdsat_get_error": [P, ctypes.POINTER(ctypes.c_uint32)],
             "sdsat_op_gemm": [P, P, I, I, P, I, P],
@@ -302,6 +305,27 @@ class Context:
         _check(_lib().sdsat_build_block(self.handle, kv.handle, mode, _ptr(prev_out), _ptr(prev_acc),
                                         _ptr(draft_table), table_stride, b, q, _ptr(tokens_out)),
                "sdsat_build_block")
+
+    # ---- tree-structured draft step 2 (Sec. 2.1.2) ----
+    def block_forward_tree(self, kv: KV, tokens, parent, logits, b: int, q: int):
+        self._bind_stream()
+        _check(_lib().sdsat_block_forward_tree(self.handle, kv.handle, _ptr(tokens), _ptr(parent), b, q,
+                                               _ptr(logits)), "sdsat_block_forward_tree")
+
+    def accept_tree(self, kv: KV, logits, tokens, parent, b: int, q: int, accepted_len, out_tokens, path=None,
+                    temperature: float = 0.0, top_p: float = 1.0, seed: int = 0, top_k: int = 0,
+                    commit: bool = True):
+        self._bind_stream()
+        _check(_lib().sdsat_accept_tree(self.handle, kv.handle, _ptr(logits), _ptr(tokens), _ptr(parent), b, q,
+                                        temperature, top_p, seed, top_k, _ptr(accepted_len), _ptr(out_tokens),
+                                        _ptr(path), int(commit)), "sdsat_accept_tree")
+
+    def build_tree_block(self, kv: KV, mode: int, prev_out, prev_q: int, prev_acc, tokens_out, b: int, k: int,
+                         draft_tables=None, width: int = 1, table_stride: int = 0):
+        self._bind_stream()
+        _check(_lib().sdsat_build_tree_block(self.handle, kv.handle, mode, _ptr(prev_out), prev_q, _ptr(prev_acc),
+                                             _ptr(draft_tables), width, table_stride, b, k, _ptr(tokens_out)),
+               "sdsat_build_tree_block")
 
     def prefill(self, kv: KV, seq: int, tokens):
         self._bind_stream()

@@ -10,6 +10,14 @@
 //
 // One CTA per block row selects that row's target; the last CTA of a sequence
 // (per-sequence counter, no waiting) runs the prefix scan and the commit.
+//
+// Tree blocks (Sec. 2.1.2): the rows are the nodes of a draft tree in
+// topological order (parent[j] < j, row 0 the root).  Row j sits at position
+// len + depth(j); a child is accepted when its parent is and its token equals
+// the parent's target, and the deepest accepted node (lowest row among equally
+// deep ones) ends the accepted path n_0 = 0, ..., n_m.  Its targets are
+// emitted, and a compaction kernel moves the path's K and V rows to the slots
+// len + 1 .. len + m before len advances by 1 + m.
 #include "common.cuh"
 #include "internal.h"
 
@@ -360,6 +368,23 @@ __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* r
   return out;
 }
 
+// parent of tree row i (0 < i < q): an earlier row; anything else is flagged and read as the root
+__device__ __forceinline__ int tree_parent(const int* par, int i, uint32_t* err) {
+  int pi = __ldcg(par + i);
+  if (pi < 0 || pi >= i) {
+    set_error(err, ERR_TREE);
+    pi = 0;
+  }
+  return pi;
+}
+
+// depth of tree row j (the root has depth 0); at most j steps since parents are earlier rows
+__device__ __forceinline__ int tree_depth(const int* par, int j, uint32_t* err) {
+  int d = 0;
+  for (int i = j; i > 0; i = tree_parent(par, i, err)) ++d;
+  return d;
+}
+
 __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams p) {
   __shared__ float redf[32];
   __shared__ uint64_t red[32];
@@ -373,7 +398,8 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
   if (p.temperature <= 0.f) {
     t = row_argmax(row, p.V, p.err, redf, redi);
   } else {
-    const int position = __ldcg(p.len + s) + j + 1;   // the produced token's position
+    // the produced token's position: one past the row's own (len + j, or len + depth(j))
+    const int position = __ldcg(p.len + s) + (p.parent ? tree_depth(p.parent + sl * p.q, j, nullptr) : j) + 1;
     t = row_nucleus(p, row, position, s, redf, red, redi);
   }
   if (threadIdx.x == 0) p.targets[sl * p.q + j] = t;
@@ -386,11 +412,42 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
   int tg[SDSAT_ATT_MAXQ];
   for (int i = 0; i < p.q; ++i) tg[i] = __ldcg(p.targets + sl * p.q + i);
   int m = 0;
-  for (int i = 1; i <= p.n_verify; ++i) {          // Eq. 3: prefix of matching drafts
-    if (__ldcg(p.drafts + sl * p.q + i) != tg[i - 1]) break;
-    m = i;
+  if (!p.parent) {
+    for (int i = 1; i <= p.n_verify; ++i) {        // Eq. 3: prefix of matching drafts
+      if (__ldcg(p.drafts + sl * p.q + i) != tg[i - 1]) break;
+      m = i;
+    }
+    for (int i = 0; i < p.q; ++i) p.out_tokens[sl * p.q + i] = tg[i];
+  } else {
+    // Sec. 2.1.2: the longest branch accepted by the chain test applied along every branch
+    const int* par = p.parent + sl * p.q;
+    int dep[SDSAT_ATT_MAXQ], path[SDSAT_ATT_MAXQ];
+    uint32_t accm = 1u;
+    int best = 0;
+    dep[0] = 0;
+    for (int i = 1; i < p.q; ++i) {
+      const int pi = tree_parent(par, i, p.err);
+      dep[i] = dep[pi] + 1;
+      if (((accm >> pi) & 1u) && __ldcg(p.drafts + sl * p.q + i) == tg[pi]) {
+        accm |= 1u << i;
+        if (dep[i] > dep[best]) best = i;
+      }
+    }
+    m = dep[best];
+    for (int d = m, i = best; d >= 0; --d) {
+      path[d] = i;
+      if (d > 0) i = tree_parent(par, i, nullptr);
+    }
+    for (int i = 0; i < p.q; ++i) {
+      p.out_tokens[sl * p.q + i] = i <= m ? tg[path[i]] : -1;
+      if (p.path) p.path[sl * p.q + i] = i <= m ? path[i] : -1;
+    }
+    // the compaction kernel's input: committed length before this step, m, the path rows
+    int* w = p.tree_ws + sl * TREE_WS_STRIDE;
+    w[0] = __ldcg(p.len + s);
+    w[1] = m;
+    for (int i = 0; i <= m; ++i) w[2 + i] = path[i];
   }
-  for (int i = 0; i < p.q; ++i) p.out_tokens[sl * p.q + i] = tg[i];
   p.accepted_len[sl] = 1 + m;
   if (p.commit) {
     const int nl = __ldcg(p.len + s) + 1 + m;
@@ -504,30 +561,93 @@ cudaError_t launch_split(const float* x, int M, int K, __nv_bfloat16* xhi, __nv_
 }
 
 // ---- block input of draft step 1 (mode 1) and draft step 2 (mode 2) --------------------
-__global__ void build_block_kernel(int mode, const int* prev_out, const int* prev_acc, const int* table,
-                                   int table_stride, const int* len, const int* adaptive, int q, int* tokens) {
+// The previous block had prev_q rows per sequence.  Mode 2 builds `width` chains of k drafts
+// below the root (width 1: the chain block; row 1 + w*k + i - 1 holds branch w's draft for
+// position len + i, from table w).
+__global__ void build_block_kernel(BuildParams b) {
   pdl_wait();
   pdl_trigger();
   const int sl = blockIdx.x, j = threadIdx.x;
-  if (j >= q) return;
+  if (j >= b.q) return;
+  const int* prev = b.prev_out + sl * b.prev_q;
   int t;
-  if (mode == 1) {
-    t = (j == 0) ? __ldcg(prev_out + sl * q + __ldcg(prev_acc + sl) - 1) : adaptive[j - 1];
+  if (b.mode == 1) {
+    t = (j == 0) ? __ldcg(prev + __ldcg(b.prev_acc + sl) - 1) : b.adaptive[j - 1];
+  } else if (j == 0) {
+    t = __ldcg(prev);
   } else {
-    if (j == 0) t = __ldcg(prev_out + sl * q);
-    else if (table) t = __ldcg(table + (size_t)sl * table_stride + __ldcg(len + sl) + j);
-    else t = __ldcg(prev_out + sl * q + j);
+    const int w = (j - 1) / b.k, i = (j - 1) % b.k + 1;
+    if (b.table)
+      t = __ldcg(b.table + ((size_t)w * b.table_batch + sl) * b.table_stride + __ldcg(b.len + sl) + i);
+    else
+      t = __ldcg(prev + i);
   }
-  tokens[sl * q + j] = t;
+  b.tokens[sl * b.q + j] = t;
 }
 
-cudaError_t launch_build_block(int mode, const int* prev_out, const int* prev_acc, const int* table,
-                               int table_stride, const int* len, const int* adaptive, int nb, int q,
-                               int* tokens_out, cudaStream_t st, bool pdl) {
+cudaError_t launch_build_block(const BuildParams& b, cudaStream_t st, bool pdl) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(nb), dim3(32), st, pdl, attr);
-  return cudaLaunchKernelEx(&cfg, build_block_kernel, mode, prev_out, prev_acc, table, table_stride, len,
-                            adaptive, q, tokens_out);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(b.nb), dim3(32), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, build_block_kernel, b);
+}
+
+// ---- tree blocks: positions and attention masks, and the commit's KV compaction ----------
+// Row j of a tree block: position len + depth(j) and the mask of the block rows it attends
+// (its ancestors and itself).  One thread per row.
+__global__ void tree_prep_kernel(const int* parent, const int* len, int nb, int q, int* pos, uint32_t* anc,
+                                 uint32_t* err) {
+  pdl_wait();
+  pdl_trigger();
+  const int r = threadIdx.x;
+  if (r >= nb * q) return;
+  const int sl = r / q, j = r % q;
+  const int* par = parent + sl * q;
+  if (j == 0 && __ldcg(par) != -1) set_error(err, ERR_TREE);
+  uint32_t m = 1u << j;
+  int d = 0;
+  for (int i = j; i > 0; ++d) {
+    i = tree_parent(par, i, err);
+    m |= 1u << i;
+  }
+  pos[r] = __ldcg(len + sl) + d;
+  anc[r] = m;
+}
+
+cudaError_t launch_tree_prep(const int* parent, const int* len, int nb, int q, int* pos, uint32_t* anc,
+                             uint32_t* err, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(1), dim3(TREE_MAX_ROWS), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, tree_prep_kernel, parent, len, nb, q, pos, anc, err);
+}
+
+// Slot len0 + i receives the K and V rows of slot len0 + n_i (i = 1..m; n_i >= i, so no
+// source is overwritten before it is read).  One CTA per (layer, head) and sequence, 16-byte
+// chunks.
+__global__ void tree_compact_kernel(const int* ws, int H, int hd, int cap, int batch, __nv_bfloat16* kc,
+                                    __nv_bfloat16* vc) {
+  pdl_wait();
+  pdl_trigger();
+  const int l = blockIdx.x / H, h = blockIdx.x % H, s = blockIdx.y;
+  const int* w = ws + s * TREE_WS_STRIDE;
+  const int len0 = __ldcg(w), m = __ldcg(w + 1);
+  const int chunks = hd / 8;   // 16-byte chunks per row
+  const size_t off = (((size_t)l * batch + s) * H + h) * cap * hd;
+  for (int x = threadIdx.x; x < 2 * m * chunks; x += blockDim.x) {
+    const int which = x / (m * chunks), rem = x % (m * chunks);
+    const int i = 1 + rem / chunks, ch = rem % chunks;
+    const int n = __ldcg(w + 2 + i);
+    if (n == i || len0 + n >= cap) continue;
+    __nv_bfloat16* base = (which ? vc : kc) + off;
+    const uint4 v = __ldcg(reinterpret_cast<const uint4*>(base + (size_t)(len0 + n) * hd) + ch);
+    __stcg(reinterpret_cast<uint4*>(base + (size_t)(len0 + i) * hd) + ch, v);
+  }
+}
+
+cudaError_t launch_tree_compact(const int* ws, int nb, int L, int H, int hd, int cap, int batch,
+                                __nv_bfloat16* k, __nv_bfloat16* v, cudaStream_t st, bool pdl) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = make_cfg(dim3(L * H, nb), dim3(64), st, pdl, attr);
+  return cudaLaunchKernelEx(&cfg, tree_compact_kernel, ws, H, hd, cap, batch, k, v);
 }
 
 // ---- explicit commit / rollback, and prefill commit --------------------------------------

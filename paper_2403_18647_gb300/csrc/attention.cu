@@ -3,8 +3,10 @@
 // In one block forward, row j of sequence s attends to the committed slots
 // [0, len[s]) and to block rows 0..j (slots len[s] .. len[s]+j), which the QKV
 // epilogue has just written; this is how Eq. 1-2 evaluate every appended
-// position of the block in one pass.  The bytes are the K and V rows (bf16,
-// hd*2 bytes each), read once per (sequence, head) for all q rows together.
+// position of the block in one pass.  A tree block (Sec. 2.1.2) replaces the
+// rows 0..j by row j's ancestors and itself, given as one bit mask per row.
+// The bytes are the K and V rows (bf16, hd*2 bytes each), read once per
+// (sequence, head) for all q rows together.
 //
 // Work is split into units of ATT_UNIT = 64 consecutive slots of one
 // (sequence, head), ordered (sequence, head, unit).  One wave of P CTAs (two
@@ -51,7 +53,8 @@ struct AttCfg {
   static constexpr size_t OFF_RED = OFF_P + 2 * 16 * PSTRIDE;                       // [16][RED]
   static constexpr size_t OFF_MERGE = OFF_RED + 16 * RED * 4;                       // ms, ls, w [16][SEG], inv [16]
   static constexpr size_t OFF_SEQ = OFF_MERGE + (3 * 16 * ATT_SEG_MAX + 16) * 4;    // len, units [64], first unit [65]
-  static constexpr size_t OFF_BAR = (OFF_SEQ + (64 + 64 + 65) * 4 + 7) / 8 * 8;
+  static constexpr size_t OFF_ANC = OFF_SEQ + (64 + 64 + 65) * 4;                   // [16] visible block rows per row
+  static constexpr size_t OFF_BAR = (OFF_ANC + 16 * 4 + 7) / 8 * 8;
   static constexpr size_t SMEM = 1024 + OFF_BAR + ATT_STAGES * 8 + 16;
 };
 
@@ -105,6 +108,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   int* len_seq = reinterpret_cast<int*>(smem + C::OFF_SEQ);     // [64] committed length of each sequence
   int* nu_seq = len_seq + 64;                                   // [64] units per head of each sequence
   int* base = nu_seq + 64;                                      // [65] first unit of each sequence
+  uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + C::OFF_ANC);   // [16] block rows row j sees (bit i)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);   // [ATT_STAGES] K and V of the stage landed
   volatile int* abort_flag = reinterpret_cast<volatile int*>(full + ATT_STAGES);
   int* s_last = reinterpret_cast<int*>(full + ATT_STAGES) + 1;
@@ -226,7 +230,9 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   for (int k = 0; k < n; ++k) {
     const int u = u0 + k;
     if (u == seg_first) {
-      // ---- a new (sequence, head): q (scaled by 1/sqrt(hd)) as bf16 hi + lo, rows >= q zero
+      // ---- a new (sequence, head): the rows' visible block rows (causal: 0..j; tree: the
+      // ancestors and the row itself), q (scaled by 1/sqrt(hd)) as bf16 hi + lo, rows >= q zero
+      if (tid < 16) anc_s[tid] = (p.anc && tid < q) ? __ldcg(p.anc + sl * q + tid) : (2u << tid) - 1u;
       for (int i = tid; i < 16 * (HD / 2); i += 128) {
         const int j = i / (HD / 2), d = (i % (HD / 2)) * 2;
         float x0 = 0.f, x1 = 0.f;
@@ -289,14 +295,15 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
         for (int e = 0; e < 4; ++e) St[t][e] += Sl[t][e];
     }
     // St[t][e] is the score of key kb + g + 8*(e >> 1) for query row t*8 + 2*tig + (e & 1).
-    // mask: row j sees key slot kp iff kp <= len + j (and kp < nkeys, j < q)
+    // mask: row j sees key slot kp iff kp < len, or kp = len + i for a block row i that
+    // anc_s[j] marks (and kp < nkeys, j < q)
 #pragma unroll
     for (int t = 0; t < QT; ++t)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int j = t * 8 + 2 * tig + (e & 1);
         const int kp = c0 + kb + g + 8 * (e >> 1);
-        if (!ok || j >= q || kp >= nkeys || kp > len + j) St[t][e] = -INFINITY;
+        if (!ok || j >= q || kp >= nkeys || (kp >= len && !((anc_s[j] >> (kp - len)) & 1u))) St[t][e] = -INFINITY;
       }
     // ---- the unit's row maxima: over the warp's lanes holding other keys (g), then the four
     // warps through shared memory; the running statistics stay in registers

@@ -19,6 +19,7 @@ enum : uint32_t {
   ERR_CAPACITY = 1u << 2,     // a block row would pass the KV capacity; not written
   ERR_TOKEN = 1u << 3,        // a token id outside [0, vocab) was read; id 0 used
   ERR_POSITION = 1u << 4,     // a RoPE position outside the table; clamped
+  ERR_TREE = 1u << 5,         // a tree row whose parent is not an earlier row; hung below the root
 };
 
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s

@@ -117,6 +117,7 @@ struct AttnParams {
   const float* Q;       // [rows][q_ld] (row = sl*q + j), head h at column h*hd
   int q_ld;
   const int* len;       // [B]
+  const uint32_t* anc;  // [nb*q] tree blocks: bit i of row j = row j attends block row i; null = causal
   int seq0, nb, q, H, hd, cap;
   float* out;           // [rows][out_ld] fp32
   int out_ld;
@@ -158,13 +159,34 @@ struct AcceptParams {
   int* targets;             // scratch [nb*q]
   int* counters;            // scratch [nb], zero between launches
   long long* emitted;       // [B] tokens emitted per sequence (commit only), or null
+  const int* parent;        // tree blocks: [nb*q] parent row of every row (row 0: -1); null = chain
+  int* path;                // tree blocks: [nb*q] accepted path rows, -1 past its end (optional)
+  int* tree_ws;             // tree blocks: [nb][TREE_WS_STRIDE] len before the step, m, path rows
   uint32_t* err;
 };
+constexpr int TREE_WS_STRIDE = SDSAT_ATT_MAXQ + 2;
+constexpr int TREE_MAX_ROWS = 64;   // rows of one block forward (the tree kernels run one thread per row)
 cudaError_t launch_accept(const AcceptParams& p, cudaStream_t st, bool pdl);
 
-cudaError_t launch_build_block(int mode, const int* prev_out, const int* prev_acc, const int* table,
-                               int table_stride, const int* len, const int* adaptive, int nb, int q,
-                               int* tokens_out, cudaStream_t st, bool pdl);
+struct BuildParams {
+  int mode;                 // 1: draft step 1 block, 2: draft step 2 block
+  const int* prev_out;      // [nb][prev_q] the previous block's emitted tokens
+  int prev_q;
+  const int* prev_acc;      // [nb] its accepted lengths
+  const int* table;         // [width][table_batch][table_stride] draft tables, or null
+  int table_stride, table_batch;
+  const int* len;           // [B] committed lengths
+  const int* adaptive;      // [SDSAT_MAX_ADAPTIVE] adaptive token ids
+  int nb, q, k;             // q rows per sequence; mode 2: q = 1 + width * k
+  int* tokens;              // [nb][q]
+};
+cudaError_t launch_build_block(const BuildParams& b, cudaStream_t st, bool pdl);
+// tree block rows: positions len + depth and the attention masks (ancestors and self)
+cudaError_t launch_tree_prep(const int* parent, const int* len, int nb, int q, int* pos, uint32_t* anc,
+                             uint32_t* err, cudaStream_t st, bool pdl);
+// move the accepted path's K / V rows to contiguous slots (input: AcceptParams::tree_ws)
+cudaError_t launch_tree_compact(const int* ws, int nb, int L, int H, int hd, int cap, int batch,
+                                __nv_bfloat16* k, __nv_bfloat16* v, cudaStream_t st, bool pdl);
 cudaError_t launch_commit(int* len, const int* new_len, int nb, int cap, uint32_t* err, cudaStream_t st,
                           bool pdl);
 cudaError_t launch_add_len(int* len, int seq, int n, int cap, uint32_t* err, cudaStream_t st, bool pdl);

@@ -21,6 +21,7 @@
 
 using namespace sdsat;
 static_assert(TRACE_WORDS == SDSAT_TRACE_WORDS, "trace record size");
+static_assert(TREE_MAX_ROWS == SDSAT_MAX_ROWS && SDSAT_ATT_MAXQ == SDSAT_MAX_Q, "tree kernel limits");
 
 namespace {
 
@@ -86,11 +87,11 @@ struct LayerMaps {
 // kernel classes for the profiling hook
 enum KClass : int {
   K_RMSNORM = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
-  K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_COUNT
+  K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_TREE_PREP, K_TREE_COMPACT, K_COUNT
 };
 const char* const KCLASS_NAME[K_COUNT] = {"rmsnorm", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
                                           "gemm_lm_head", "accept", "build_block", "kv_commit", "prefill_commit",
-                                          "gemm_op", "attention_op"};
+                                          "gemm_op", "attention_op", "tree_prep", "tree_compact"};
 
 constexpr int MAX_GEMM_TILES = 1 << 16;
 constexpr int OP_MAX_K = 32768;   // K limit of sdsat_op_gemm (its operand scratch is sized at create)
@@ -125,6 +126,9 @@ struct sdsat_ctx {
   int* att_counters = nullptr;
   int* acc_targets = nullptr;
   int* acc_counters = nullptr;
+  int* tree_pos = nullptr;     // [SDSAT_MAX_ROWS] tree block positions (len + depth)
+  uint32_t* tree_anc = nullptr;   // [SDSAT_MAX_ROWS] tree block attention masks
+  int* tree_ws = nullptr;      // [SDSAT_MAX_ROWS][TREE_WS_STRIDE] tree commit: len, m, path
   int* adaptive = nullptr;
   uint32_t* err = nullptr;
   __nv_bfloat16* x_hi[X_COUNT] = {};
@@ -232,9 +236,9 @@ void set_plain(GemmParams& g, const CUtensorMap& m, int N, int K) {
   g.kc = (K + 63) / 64;
 }
 
-// one block forward of sequences seq0 .. seq0+nb-1, q rows each
+// one block forward of sequences seq0 .. seq0+nb-1, q rows each (anc: tree attention masks)
 sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const int32_t* tokens,
-                     const int32_t* positions, float* logits) {
+                     const int32_t* positions, float* logits, const uint32_t* anc = nullptr) {
   const sdsat_config& cf = c->cfg;
   const int M = nb * q, d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd, L = cf.n_layers;
   cudaStream_t st = c->stream;
@@ -362,6 +366,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.Q = c->qbuf;
     a.q_ld = R;
     a.len = kv->len;
+    a.anc = anc;
     a.seq0 = seq0;
     a.nb = nb;
     a.q = q;
@@ -390,7 +395,7 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
 
 sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, const int32_t* drafts, int b, int q,
                            int n_verify, float top_p, float temperature, uint64_t seed, int top_k, int32_t* acc,
-                           int32_t* out, int commit) {
+                           int32_t* out, int commit, const int32_t* parent = nullptr, int32_t* path = nullptr) {
   if (!c || !kv || kv->ctx != c || !logits || !drafts || !acc || !out) return SDSAT_EINVAL;
   if (b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
   if (n_verify < 0 || n_verify >= q || top_k < 0) return SDSAT_EINVAL;
@@ -420,8 +425,18 @@ sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, cons
   p.counters = c->acc_counters;
   p.err = c->err;
   p.emitted = kv->emitted;
-  return timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, c->pdl); }) == cudaSuccess ? SDSAT_OK
-                                                                                          : SDSAT_ECUDA;
+  p.parent = parent;
+  p.path = path;
+  p.tree_ws = c->tree_ws;
+  if (timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+  if (!parent) return SDSAT_OK;
+  const sdsat_config& cf = c->cfg;
+  return timed(c, K_TREE_COMPACT, [&] {
+           return launch_tree_compact(c->tree_ws, b, cf.n_layers, cf.n_heads, cf.head_dim, kv->cap, kv->batch, kv->k,
+                                      kv->v, c->stream, c->pdl);
+         }) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
 }
 
 }  // namespace
@@ -519,6 +534,8 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
             dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * ATT_SEG_MAX * 2) &&
             dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
+            dalloc(c, &c->tree_pos, rows) && dalloc(c, &c->tree_anc, rows) &&
+            dalloc(c, &c->tree_ws, (size_t)rows * TREE_WS_STRIDE) &&
             dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)rows * OP_MAX_K) &&
             dalloc(c, &c->ssq, (size_t)rows * ((d + 127) / 128)) &&
             dalloc(c, &c->xop_lo, (size_t)rows * OP_MAX_K);
@@ -665,6 +682,17 @@ sdsat_status sdsat_block_forward(sdsat_ctx* c, sdsat_kv* kv, const int32_t* toke
   return forward(c, kv, 0, b, q, tokens_dev, positions_dev, logits_dev);
 }
 
+sdsat_status sdsat_block_forward_tree(sdsat_ctx* c, sdsat_kv* kv, const int32_t* tokens_dev,
+                                      const int32_t* parent_dev, int b, int q, float* logits_dev) {
+  if (!c || !kv || kv->ctx != c || !c->has_weights || !tokens_dev || !parent_dev || !logits_dev) return SDSAT_EINVAL;
+  if (b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
+  if (timed(c, K_TREE_PREP, [&] {
+        return launch_tree_prep(parent_dev, kv->len, b, q, c->tree_pos, c->tree_anc, c->err, c->stream, c->pdl);
+      }) != cudaSuccess)
+    return SDSAT_ECUDA;
+  return forward(c, kv, 0, b, q, tokens_dev, c->tree_pos, logits_dev, c->tree_anc);
+}
+
 sdsat_status sdsat_prefill(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* tokens_dev, int n) {
   if (!c || !kv || kv->ctx != c || !c->has_weights || !tokens_dev || seq < 0 || seq >= kv->batch || n < 0)
     return SDSAT_EINVAL;
@@ -692,6 +720,15 @@ sdsat_status sdsat_accept_nucleus(sdsat_ctx* c, sdsat_kv* kv, const float* logit
                                   int top_k, int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit) {
   return accept_common(c, kv, logits_dev, drafts_dev, b, q, n_verify, top_p, temperature, rng_seed, top_k,
                        accepted_len_dev, out_tokens_dev, commit);
+}
+
+sdsat_status sdsat_accept_tree(sdsat_ctx* c, sdsat_kv* kv, const float* logits_dev, const int32_t* tokens_dev,
+                               const int32_t* parent_dev, int b, int q, float temperature, float top_p,
+                               uint64_t rng_seed, int top_k, int32_t* accepted_len_dev, int32_t* out_tokens_dev,
+                               int32_t* path_dev, int commit) {
+  if (!parent_dev || !(temperature >= 0.f)) return SDSAT_EINVAL;
+  return accept_common(c, kv, logits_dev, tokens_dev, b, q, q - 1, temperature > 0.f ? top_p : 1.f,
+                       temperature, rng_seed, top_k, accepted_len_dev, out_tokens_dev, commit, parent_dev, path_dev);
 }
 
 sdsat_status sdsat_kv_commit(sdsat_ctx* c, sdsat_kv* kv, const int32_t* new_len_dev, int b) {
@@ -807,10 +844,28 @@ sdsat_status sdsat_build_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32
   if ((mode != 1 && mode != 2) || b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q) return SDSAT_EINVAL;
   if (mode == 1 && c->cfg.n_adaptive > 1 && q - 1 > c->cfg.n_adaptive) return SDSAT_EINVAL;
   if (draft_table_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
-  return timed(c, K_BUILD_BLOCK, [&] {
-           return launch_build_block(mode, prev_out_dev, prev_acc_dev, draft_table_dev, table_stride, kv->len,
-                                     c->adaptive, b, q, tokens_out_dev, c->stream, c->pdl);
-         }) == cudaSuccess
+  BuildParams bp{mode, prev_out_dev, q, prev_acc_dev, draft_table_dev, table_stride, kv->batch, kv->len,
+                 c->adaptive, b, q, q - 1, tokens_out_dev};
+  return timed(c, K_BUILD_BLOCK, [&] { return launch_build_block(bp, c->stream, c->pdl); }) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_build_tree_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const int32_t* prev_out_dev, int prev_q,
+                                    const int32_t* prev_acc_dev, const int32_t* draft_tables_dev, int width,
+                                    int table_stride, int b, int k, int32_t* tokens_out_dev) {
+  if (!c || !kv || kv->ctx != c || !prev_out_dev || !prev_acc_dev || !tokens_out_dev) return SDSAT_EINVAL;
+  if ((mode != 1 && mode != 2) || b < 1 || b > kv->batch || k < 1 || width < 1 || prev_q < 1 ||
+      prev_q > SDSAT_MAX_Q)
+    return SDSAT_EINVAL;
+  const int q = mode == 1 ? k + 1 : 1 + width * k;
+  if (q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
+  if (mode == 1 && c->cfg.n_adaptive > 1 && k > c->cfg.n_adaptive) return SDSAT_EINVAL;
+  if (mode == 2 && !draft_tables_dev && (width > 1 || k >= prev_q)) return SDSAT_EINVAL;
+  if (draft_tables_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
+  BuildParams bp{mode, prev_out_dev, prev_q, prev_acc_dev, draft_tables_dev, table_stride, kv->batch, kv->len,
+                 c->adaptive, b, q, k, tokens_out_dev};
+  return timed(c, K_BUILD_BLOCK, [&] { return launch_build_block(bp, c->stream, c->pdl); }) == cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;
 }

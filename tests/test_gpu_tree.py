@@ -1,0 +1,377 @@
+"""Parity of the tree-structured draft step 2 (Sec. 2.1.2) on the GPU against oracle/tree.py.
+
+  * tree forward: logits and the K / V rows written at slots len + j (rotated at
+    position len + depth(j)) against the oracle's tree forward, within the chain
+    step's tolerances; a chain-shaped tree reproduces sdsat_block_forward exactly;
+  * tree acceptance on given logits: targets, the accepted path, the emitted
+    tokens, accepted lengths and the committed lengths bit-exact, greedy and
+    nucleus, several tree shapes and b = 2;
+  * compaction: the path's K / V rows land in slots len + 1 .. len + m bit-exact;
+  * the whole tree loop teacher-forced against the oracle's tree decode, and run
+    on the device alone it emits the plain greedy sequence (greedy invariant).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import decode as OD
+from oracle import model as OM
+from oracle import sampling as OS
+from oracle import tree as OT
+
+pytestmark = pytest.mark.gpu
+
+K = 3
+WIDTH = 2
+PROMPT = 96
+N_NEW = 40
+LOGIT_MAX_ABS = 3e-2
+LOGIT_REL_RMS = 1e-2
+TIE_GAP = 1e-2
+
+# an irregular tree: branching at several depths, siblings interleaved with cousins
+IRREGULAR = [-1, 0, 0, 1, 2, 1, 3, 3, 6, 4, 0]
+TREES = [OT.chains_parent(WIDTH, K), IRREGULAR, OT.chains_parent(3, 5), [-1]]
+
+
+@pytest.fixture(scope="module")
+def sd():
+    import paper_2403_18647_gb300 as sd
+    return sd
+
+
+@pytest.fixture(scope="module")
+def tiny(sd):
+    shape = synth.SHAPES["tiny"]
+    w_gpu = synth.make_model(shape, seed=0, device="cuda", gain_std=0.1)
+    w_cpu = synth.make_model(shape, seed=0, device="cpu", gain_std=0.1)
+    ctx = sd.Context(shape, w_gpu, max_position=1024)
+    return shape, ctx, OM.Weights(shape, tensors=w_cpu)
+
+
+def _i32(x):
+    return torch.tensor(list(x), dtype=torch.int32, device="cuda")
+
+
+def _compare_logits(got, ref):
+    err = np.abs(got - ref).max()
+    rel = np.sqrt(((got - ref) ** 2).mean() / (ref ** 2).mean())
+    assert err <= LOGIT_MAX_ABS and rel <= LOGIT_REL_RMS, (err, rel)
+
+
+@pytest.mark.parametrize("parent", TREES[:3], ids=["chains2x3", "irregular", "chains3x5"])
+def test_tree_forward_matches_oracle(sd, tiny, parent):
+    shape, ctx, W = tiny
+    q = len(parent)
+    lens = [37, 70]
+    b = len(lens)
+    kv = ctx.kv(b, 128)
+    kvo = OM.KVCache(shape, b, 128)
+    for s in range(b):
+        p = synth.prompt_ids(0, 20 + s, lens[s], 4096)
+        ctx.prefill(kv, s, p.cuda())
+        OM.prefill(W, kvo, s, p.tolist())
+    toks = synth.uniform_ids(0, 77, b * q, shape.vocab)
+    lg = torch.empty(b * q, shape.vocab, device="cuda")
+    ctx.block_forward_tree(kv, toks.cuda(), _i32(parent * b), lg, b, q)
+    got = lg.cpu().numpy().astype(np.float64)
+    for s in range(b):
+        ref = OT.tree_forward(W, kvo, s, toks[s * q:(s + 1) * q].tolist(), parent)
+        _compare_logits(got[s * q:(s + 1) * q], ref)
+        for l in range(shape.n_layers):
+            k, v = ctx.kv_read(kv, l, s, lens[s], q)
+            rk, rv = kvo.K[l][s][:, lens[s]:lens[s] + q], kvo.V[l][s][:, lens[s]:lens[s] + q]
+            scale = max(np.abs(rk).max(), np.abs(rv).max())
+            assert np.abs(k.float().cpu().numpy() - rk).max() <= 2e-2 * scale
+            assert np.abs(v.float().cpu().numpy() - rv).max() <= 2e-2 * scale
+    assert ctx.kv_lengths(kv).cpu().tolist() == lens   # the forward commits nothing
+    assert ctx.get_error() == 0
+
+
+def test_chain_tree_is_the_block_forward(sd, tiny):
+    """parent[j] = j - 1 gives the block-causal mask and positions len + j: the same logits, bit for bit."""
+    shape, ctx, W = tiny
+    q = 6
+    toks = synth.uniform_ids(0, 78, 2 * q, shape.vocab).cuda()
+    outs = []
+    for tree in (True, False):
+        kv = ctx.kv(2, 96)
+        for s in range(2):
+            ctx.prefill(kv, s, synth.prompt_ids(0, 30 + s, 50 + 7 * s, 4096).cuda())
+        lg = torch.empty(2 * q, shape.vocab, device="cuda")
+        if tree:
+            ctx.block_forward_tree(kv, toks, _i32(list(range(-1, q - 1)) * 2), lg, 2, q)
+        else:
+            ctx.block_forward(kv, toks, lg, 2, q)
+        outs.append(lg)
+    assert torch.equal(outs[0], outs[1])
+
+
+def _accept_case(shape, parent, b, lens, sp, seed):
+    """Random logits and tokens; roughly half of the non-root rows copy their parent's target,
+    so branches of several lengths are accepted."""
+    q = len(parent)
+    g = torch.Generator().manual_seed(seed)
+    logits = (torch.randn(b * q, shape.vocab, generator=g) * 3.0).float()
+    d = OT.depths(parent)
+    tokens = torch.randint(0, shape.vocab, (b * q,), generator=g, dtype=torch.int32)
+    for s in range(b):
+        t = [OS.select(logits[s * q + j].numpy(), sp.temperature, sp.top_p, sp.seed, lens[s] + d[j] + 1, s,
+                       sp.top_k)[0] for j in range(q)]
+        for j in range(1, q):
+            if torch.rand(1, generator=g).item() < 0.6:
+                tokens[s * q + j] = t[parent[j]]
+    return logits, tokens
+
+
+@pytest.mark.parametrize("temperature", [0.0, 0.2, 1.0])
+@pytest.mark.parametrize("parent", TREES, ids=["chains2x3", "irregular", "chains3x5", "root"])
+def test_tree_accept_matches_oracle(sd, tiny, parent, temperature):
+    shape, ctx, W = tiny
+    q, b = len(parent), 2
+    lens = [21, 58]
+    sp = OD.SamplingParams(temperature, 0.95 if temperature > 0 else 1.0, 10 if temperature == 1.0 else 0,
+                           seed=99)
+    kv = ctx.kv(b, 96)
+    for s in range(b):
+        ctx.prefill(kv, s, synth.prompt_ids(0, 40 + s, lens[s], 4096).cuda())
+    # known K / V rows in the block's slots, to check the compaction
+    Hd = (shape.n_heads, q, shape.head_dim)
+    rows = {}
+    for l in range(shape.n_layers):
+        for s in range(b):
+            kr = synth.kv_values(s, l, 0, Hd).cuda()
+            vr = synth.kv_values(s, l, 1, Hd).cuda()
+            ctx.kv_write(kv, l, s, lens[s], kr, vr)
+            rows[l, s] = (kr.cpu(), vr.cpu())
+    before = {(l, s): ctx.kv_read(kv, l, s, 0, lens[s]) for l in range(shape.n_layers) for s in range(b)}
+    for trial in range(4):
+        logits, tokens = _accept_case(shape, parent, b, lens, sp, 1000 * trial + q)
+        acc = torch.zeros(b, dtype=torch.int32, device="cuda")
+        out = torch.zeros(b * q, dtype=torch.int32, device="cuda")
+        path = torch.zeros(b * q, dtype=torch.int32, device="cuda")
+        ctx.kv_commit(kv, _i32(lens), b)
+        for l in range(shape.n_layers):
+            for s in range(b):
+                ctx.kv_write(kv, l, s, lens[s], rows[l, s][0].cuda(), rows[l, s][1].cuda())
+        ctx.accept_tree(kv, logits.cuda(), tokens.cuda(), _i32(parent * b), b, q, acc, out, path,
+                        temperature=sp.temperature, top_p=sp.top_p, seed=sp.seed, top_k=sp.top_k, commit=True)
+        got_out, got_path, got_acc = out.cpu().tolist(), path.cpu().tolist(), acc.cpu().tolist()
+        new_len = ctx.kv_lengths(kv).cpu().tolist()
+        for s in range(b):
+            t = OT.tree_targets(logits[s * q:(s + 1) * q].numpy(), sp, parent, lens[s], s)
+            ref_path = OT.tree_verify(t, tokens[s * q:(s + 1) * q].tolist(), parent)
+            m = len(ref_path) - 1
+            assert got_acc[s] == 1 + m
+            assert got_path[s * q:(s + 1) * q] == ref_path + [-1] * (q - 1 - m)
+            assert got_out[s * q:(s + 1) * q] == [t[n] for n in ref_path] + [-1] * (q - 1 - m)
+            assert new_len[s] == lens[s] + 1 + m
+            for l in range(shape.n_layers):
+                k, v = ctx.kv_read(kv, l, s, lens[s], 1 + m)
+                kr, vr = rows[l, s]
+                assert torch.equal(k.cpu(), kr[:, ref_path]) and torch.equal(v.cpu(), vr[:, ref_path])
+                k0, v0 = ctx.kv_read(kv, l, s, 0, lens[s])
+                assert torch.equal(k0, before[l, s][0]) and torch.equal(v0, before[l, s][1])
+    assert ctx.get_error() == 0
+
+
+def test_tree_accept_without_commit_leaves_lengths(sd, tiny):
+    shape, ctx, W = tiny
+    parent = IRREGULAR
+    q = len(parent)
+    kv = ctx.kv(1, 64)
+    ctx.prefill(kv, 0, synth.prompt_ids(0, 50, 30, 4096).cuda())
+    sp = OD.SamplingParams()
+    logits, tokens = _accept_case(shape, parent, 1, [30], sp, 7)
+    acc = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.zeros(q, dtype=torch.int32, device="cuda")
+    em0 = ctx.kv_emitted(kv).item()
+    ctx.accept_tree(kv, logits.cuda(), tokens.cuda(), _i32(parent), 1, q, acc, out, commit=False)
+    assert ctx.kv_lengths(kv).item() == 30
+    assert ctx.kv_emitted(kv).item() == em0
+    t = OT.tree_targets(logits.numpy(), sp, parent, 30, 0)
+    assert acc.item() == len(OT.tree_verify(t, tokens.tolist(), parent))
+
+
+def test_invalid_parent_sets_the_tree_bit(sd, tiny):
+    """A parent that is not an earlier row is read as the root and reported (no fault)."""
+    shape, ctx, W = tiny
+    kv = ctx.kv(1, 64)
+    ctx.prefill(kv, 0, synth.prompt_ids(0, 51, 20, 4096).cuda())
+    lg = torch.empty(4, shape.vocab, device="cuda")
+    ctx.block_forward_tree(kv, _i32([1, 2, 3, 4]), _i32([-1, 0, 3, 1]), lg, 1, 4)
+    assert ctx.get_error() == 0x20   # SDSAT_DEV_TREE, and nothing else
+    # the same tree with the bad entry replaced by the root
+    ctx.block_forward_tree(kv, _i32([1, 2, 3, 4]), _i32([-1, 0, 0, 1]), lg, 1, 4)
+    assert ctx.get_error() == 0
+
+
+def _oracle_tree_run(shape, W, sp, widths_match=(0.7, 0.5), n_new=N_NEW):
+    prompt = synth.prompt_ids(0, 0, PROMPT, 4096)
+    cap = PROMPT + 2 * n_new + 4 * (1 + WIDTH * K)
+    kv = OM.KVCache(shape, 1, cap)
+    OM.prefill(W, kv, 0, prompt[:-1].tolist())
+    base = kv.copy()
+    ref = OD.plain_decode(W, kv.copy(), 0, int(prompt[-1]), n_new + 2 * K + 4, sp)
+    full = torch.zeros(cap + 64, dtype=torch.int32)
+    full[PROMPT:PROMPT + len(ref)] = torch.tensor(ref, dtype=torch.int32)
+    tables = [synth.stub_table(w, 0, full, widths_match[w], shape.vocab) for w in range(WIDTH)]
+    res = OT.tree_decode(W, base.copy(), 0, int(prompt[-1]), n_new, K, WIDTH, [shape.adaptive_id], sp,
+                         [t.numpy() for t in tables], log=True)
+    return prompt, ref, tables, res, cap
+
+
+@pytest.mark.parametrize("temperature", [0.0, 0.2])
+def test_tree_loop_teacher_forced(sd, tiny, temperature):
+    """Every step of the oracle's tree decode, replayed on the GPU from the oracle's committed state."""
+    shape, ctx, W = tiny
+    sp = OD.SamplingParams(temperature, 0.95 if temperature > 0 else 1.0, 10 if temperature > 0 else 0, seed=1234)
+    prompt, ref, tables, res, cap = _oracle_tree_run(shape, W, sp)
+    parent = OT.chains_parent(WIDTH, K)
+    kv = ctx.kv(1, cap)
+    ctx.prefill(kv, 0, prompt[:-1].cuda())
+    flips = 0
+    n_tree_steps = 0
+    for st in res.steps:
+        q = len(st.tokens)
+        toks = _i32(st.tokens)
+        logits = torch.empty(q, shape.vocab, device="cuda")
+        acc = torch.empty(1, dtype=torch.int32, device="cuda")
+        out = torch.empty(q, dtype=torch.int32, device="cuda")
+        ctx.kv_commit(kv, _i32([st.len_before]), 1)
+        if st.mode == "draft":
+            ctx.block_forward(kv, toks, logits, 1, q)
+            ctx.accept_nucleus(kv, logits, toks, 1, q, 0, sp.top_p, sp.temperature, sp.seed, acc, out,
+                               top_k=sp.top_k, commit=False)
+            tg = out.cpu().tolist()
+        else:
+            n_tree_steps += 1
+            ctx.block_forward_tree(kv, toks, _i32(parent), logits, 1, q)
+            path = torch.empty(q, dtype=torch.int32, device="cuda")
+            ctx.accept_tree(kv, logits, toks, _i32(parent), 1, q, acc, out, path, temperature=sp.temperature,
+                            top_p=sp.top_p, seed=sp.seed, top_k=sp.top_k, commit=False)
+        lg = logits.cpu().numpy()
+        _compare_logits(lg.astype(np.float64), st.logits)
+        if st.mode == "draft":
+            for j in range(q):
+                if tg[j] != st.targets[j]:
+                    assert OS.top2_gap(st.logits[j]) < TIE_GAP or sp.temperature > 0
+                    flips += 1
+        else:
+            # the acceptance is bit-exact on the logits the GPU produced
+            t = OT.tree_targets(lg, sp, parent, st.len_before, 0)
+            p_ref = OT.tree_verify(t, st.tokens, parent)
+            assert acc.item() == len(p_ref)
+            assert path.cpu().tolist()[:len(p_ref)] == p_ref
+            if t != list(st.targets):
+                flips += 1
+            elif flips == 0:
+                assert acc.item() == st.accepted
+    assert n_tree_steps >= 5
+    assert flips <= (1 if temperature == 0 else len(res.steps))
+    assert ctx.get_error() == 0
+
+
+def test_tree_device_loop_equals_plain_greedy(sd, tiny):
+    """build_tree_block -> forward -> accept on the device alone: the tree loop emits the plain
+    greedy sequence (greedy invariant), and the tree accepts at least as much as its first branch."""
+    shape, ctx, W = tiny
+    sp = OD.SamplingParams()
+    prompt, ref, tables, res, cap = _oracle_tree_run(shape, W, sp)
+    stride = cap + 32
+    tab = torch.zeros(WIDTH, 1, stride, dtype=torch.int32)
+    for w in range(WIDTH):
+        n = min(stride, tables[w].numel())
+        tab[w, 0, :n] = tables[w][:n]
+    tab = tab.cuda()
+    q1, q2 = K + 1, 1 + WIDTH * K
+    parent = _i32(OT.chains_parent(WIDTH, K))
+    kv = ctx.kv(1, cap)
+    ctx.prefill(kv, 0, prompt[:-1].cuda())
+    logits = torch.empty(q2, shape.vocab, device="cuda")
+    acc = torch.ones(1, dtype=torch.int32, device="cuda")
+    out = torch.zeros(q2, dtype=torch.int32, device="cuda")
+    out[0] = int(prompt[-1])
+    toks = torch.empty(q2, dtype=torch.int32, device="cuda")
+    emitted, per_loop = [], []
+    prev_q = q2
+    while len(emitted) < N_NEW:
+        ctx.build_tree_block(kv, 1, out, prev_q, acc, toks, 1, K)
+        ctx.block_forward(kv, toks, logits, 1, q1)
+        ctx.accept_greedy(kv, logits, toks, 1, q1, 0, acc, out)
+        a1 = int(acc.item())
+        emitted += out[:a1].cpu().tolist()
+        ctx.build_tree_block(kv, 2, out, q1, acc, toks, 1, K, draft_tables=tab, width=WIDTH, table_stride=stride)
+        ctx.block_forward_tree(kv, toks, parent, logits, 1, q2)
+        ctx.accept_tree(kv, logits, toks, parent, 1, q2, acc, out)
+        a2 = int(acc.item())
+        emitted += out[:a2].cpu().tolist()
+        per_loop.append(a1 + a2)
+        prev_q = q2
+    assert all(2 <= n <= K + 2 for n in per_loop)
+    # no near-tie flip inside the generation: the same loops as the oracle's tree decode
+    assert per_loop[:-1] == res.per_loop[:len(per_loop) - 1] or emitted[:N_NEW] != ref[:N_NEW]
+    emitted = emitted[:N_NEW]
+    first_diff = next((i for i, (a, b) in enumerate(zip(emitted, ref)) if a != b), None)
+    assert first_diff is None or first_diff > 8, (first_diff, emitted[:10], ref[:10])
+    assert ctx.get_error() == 0
+
+
+def test_tree_full_size_7b(sd):
+    """7B shape, context 2047, the bench's tree (two chains of k = 5 drafts, q = 11), properties
+    that hold at any size: every tree row equals the same row of a chain block forward of its
+    root path; a greedy branch accepted to depth 3 emits the plain greedy tokens, and after the
+    compaction and commit the cache continues the plain greedy sequence."""
+    shape = synth.SHAPES["7b"]
+    k, P = 5, 2048
+    w = synth.make_model(shape, seed=0, device="cuda")
+    ctx = sd.Context(shape, w, max_position=P + 64)
+    prompt = synth.prompt_ids(0, 0, P, shape.adaptive_id).cuda()
+    kv = ctx.kv(1, P + 32)
+    ctx.prefill(kv, 0, prompt[:-1].contiguous())
+    L0 = P - 1
+    root = int(prompt[-1])
+    # plain greedy continuation g_1 .. g_5 (q = 1 forwards), then roll back
+    lg1 = torch.empty(1, shape.vocab, device="cuda")
+    acc = torch.empty(1, dtype=torch.int32, device="cuda")
+    tok = torch.tensor([root], dtype=torch.int32, device="cuda")
+    g, gaps = [], []
+    for _ in range(5):
+        ctx.block_forward(kv, tok, lg1, 1, 1)
+        row = lg1[0].cpu().numpy()
+        gaps.append(OS.top2_gap(row))
+        ctx.accept_greedy(kv, lg1, tok, 1, 1, 0, acc, tok)
+        g.append(int(tok.item()))
+    ctx.kv_commit(kv, _i32([L0]), 1)
+    if min(gaps) < TIE_GAP:
+        pytest.skip("near-tie in the plain greedy continuation")
+    wrong = [(x + 1) % shape.adaptive_id for x in g]
+    drafts = [[wrong[0]] + g[1:5], [g[0], g[1], g[2], wrong[3], wrong[4]]]   # branch 0 fails at depth 1
+    parent = OT.chains_parent(2, k)
+    q2 = len(parent)
+    toks = _i32([root] + drafts[0] + drafts[1])
+    lt = torch.empty(q2, shape.vocab, device="cuda")
+    ctx.block_forward_tree(kv, toks, _i32(parent), lt, 1, q2)
+    tree_logits = lt.clone()
+    # each branch as a chain block from the same committed state
+    lc = torch.empty(k + 1, shape.vocab, device="cuda")
+    for br in range(2):
+        ctx.block_forward(kv, _i32([root] + drafts[br]), lc, 1, k + 1)
+        rows = [0] + [1 + br * k + i for i in range(k)]
+        diff = (tree_logits[rows] - lc).abs().max().item()
+        assert diff <= LOGIT_MAX_ABS, (br, diff)
+    # the tree step proper: forward again (the chain forwards overwrote the block's slots), accept
+    ctx.block_forward_tree(kv, toks, _i32(parent), lt, 1, q2)
+    out = torch.empty(q2, dtype=torch.int32, device="cuda")
+    path = torch.empty(q2, dtype=torch.int32, device="cuda")
+    ctx.accept_tree(kv, lt, toks, _i32(parent), 1, q2, acc, out, path)
+    assert acc.item() == 4
+    assert path.cpu().tolist()[:4] == [0, 1 + k, 2 + k, 3 + k]
+    assert out.cpu().tolist()[:4] == g[:4]
+    assert ctx.kv_lengths(kv).item() == L0 + 4
+    # the compacted cache continues the plain greedy sequence: g_4 at position L0 + 4 -> g_5
+    ctx.block_forward(kv, _i32([g[3]]), lg1, 1, 1)
+    ctx.accept_greedy(kv, lg1, _i32([g[3]]), 1, 1, 0, acc, tok)
+    assert int(tok.item()) == g[4]
+    assert ctx.get_error() == 0
