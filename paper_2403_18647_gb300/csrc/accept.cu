@@ -281,13 +281,207 @@ __device__ __forceinline__ int nth_id(const uint32_t (&W)[ACC_EPT], int base, co
   return out;
 }
 
+// ---- the sampler on a compacted list ----------------------------------------------------
+// The kept set is a prefix of the order (W desc, id asc), so it lies among the heaviest
+// weights.  With a floor F such that the elements with W >= F provably contain it (top-k:
+// at least k of them, or all non-zero weights; top-p alone: their mass reaches the top-p
+// threshold), those elements are copied in ascending id order into shared memory and one
+// warp runs the same selection on them: searches cost O(list / 32) per step and no block
+// barrier.  Otherwise the block-wide searches over all ids run.
+constexpr int NUC_LIST_MAX = 2048;
+constexpr int NUC_FLOORS = 7;
+// floor f: 2^24 (the largest weight), 2^22, 2^20, 2^18, 2^16 (ratio 2^-8), 2^8 (2^-16), then 1
+// (every non-zero weight).  Weights of bucket b (nuc_bucket) are >= the floors f >= b.
+__device__ __forceinline__ uint32_t nuc_floor(int f) { return f < 5 ? 1u << (24 - 2 * f) : (f == 5 ? 256u : 1u); }
+__device__ __forceinline__ int nuc_bucket(uint32_t w) {
+  if (w == 0) return NUC_FLOORS;
+  const int e = 31 - __clz(w);
+  return e >= 16 ? (25 - e) >> 1 : (e >= 8 ? 5 : 6);
+}
+
+struct NucList {
+  uint32_t w[NUC_LIST_MAX];
+  int id[NUC_LIST_MAX];
+  uint32_t cnt[NUC_FLOORS];                 // block totals: weights >= floor f
+  unsigned long long mhi[3], mlo[3];        // masses >= floors 4, 5, 6: sum(w >> 12), sum(w & 4095)
+  int pick;
+};
+
+// warp-wide sums: per-lane values below 2^31 (counts, or weights of <= 64 list elements)
+__device__ __forceinline__ uint64_t warp_sum_w(uint32_t v) {
+  const uint32_t hi = __reduce_add_sync(0xffffffffu, v >> 16), lo = __reduce_add_sync(0xffffffffu, v & 0xFFFFu);
+  return ((uint64_t)hi << 16) + lo;
+}
+
+// over the list: sum of W (COUNT: number of elements) of those with pred(W, id)
+template <bool COUNT, typename F>
+__device__ __forceinline__ uint64_t list_sum(const NucList& L, int n, F&& pred) {
+  uint32_t s = 0;
+  for (int i = (int)(threadIdx.x & 31); i < n; i += 32) {
+    const uint32_t w = L.w[i];
+    if (pred(w, L.id[i])) s += COUNT ? 1u : w;
+  }
+  return warp_sum_w(s);
+}
+
+// largest x in [0, 2^24] with list_sum(pred_x) >= need, pred_x(w, id) = sel(w, id) && w >= x
+template <bool COUNT, typename F>
+__device__ __forceinline__ uint32_t list_threshold(const NucList& L, int n, uint64_t need, F&& sel) {
+  uint32_t lo = 0, hi = 1u << 24;
+  while (lo < hi) {
+    const uint32_t mid = lo + (hi - lo + 1) / 2;
+    if (list_sum<COUNT>(L, n, [&](uint32_t w, int id) { return w >= mid && sel(w, id); }) >= need) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// id of the r-th (r >= 1) list element, in list (= ascending id) order, with pred(W, id)
+template <typename F>
+__device__ __forceinline__ int list_nth(const NucList& L, int n, uint64_t r, F&& pred) {
+  const int lane = threadIdx.x & 31;
+  uint64_t seen = 0;
+  for (int b = 0; b < n; b += 32) {
+    const int i = b + lane;
+    const bool hit = i < n && pred(L.w[i], L.id[i]);
+    const uint32_t m = __ballot_sync(0xffffffffu, hit);
+    const uint32_t c = __popc(m);
+    if (seen + c >= r) {
+      const int k = (int)(r - seen);      // the k-th set bit of m
+      uint32_t mm = m;
+      for (int t = 1; t < k; ++t) mm &= mm - 1;
+      return __shfl_sync(0xffffffffu, L.id[b + __ffs(mm) - 1 < n ? b + __ffs(mm) - 1 : 0], 0);
+    }
+    seen += c;
+  }
+  return 0x7FFFFFFF;
+}
+
+__device__ __forceinline__ uint64_t nuc_key(uint32_t w, int id) {   // larger: heavier, then lower id
+  return ((uint64_t)w << 32) | (uint32_t)(0x7FFFFFFF - id);
+}
+
+// Steps 4-7 on the list (warp 0) when the candidates (top-k, k <= 32) or, without top-k, the
+// kept prefix have at most 32 elements: up to 32 rounds of "largest key below the previous
+// one" put them on the lanes in (W desc, id asc) order.  Returns -1 when this does not apply.
+__device__ int list_small(const AcceptParams& p, const NucList& L, int n, uint64_t S_all, bool topk, uint64_t rnd) {
+  const int lane = threadIdx.x & 31;
+  if (topk && p.top_k > 32) return -1;
+  uint64_t thr = 0;
+  if (!topk) {
+    const uint64_t prod = (uint64_t)p.p_fixed * S_all;
+    thr = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
+  }
+  const int rounds = topk ? min(p.top_k, n) : min(32, n);
+  uint64_t prev = ~0ull, mine = 0, C = 0;
+  int nc = 0;
+  bool done = topk;
+  for (int r = 0; r < rounds && !(nc > 0 && !topk && C >= thr); ++r) {
+    uint64_t best = 0;
+    for (int i = lane; i < n; i += 32) {
+      const uint64_t k = nuc_key(L.w[i], L.id[i]);
+      if (k < prev && k > best) best = k;
+    }
+    const uint32_t hi = __reduce_max_sync(0xffffffffu, (uint32_t)(best >> 32));
+    const uint32_t lo = __reduce_max_sync(0xffffffffu, (uint32_t)(best >> 32) == hi ? (uint32_t)best : 0u);
+    prev = ((uint64_t)hi << 32) | lo;
+    if (lane == r) mine = prev;
+    ++nc;
+    C += hi;   // the round's weight
+  }
+  if (!topk) done = C >= thr;   // the kept prefix: the first nc elements reach the threshold
+  if (!done) return -1;
+  const uint32_t w = lane < nc ? (uint32_t)(mine >> 32) : 0u;
+  const int id = 0x7FFFFFFF - (int)(uint32_t)mine;
+  bool kept = lane < nc;
+  if (topk) {
+    // candidates = the nc lanes; kept = the shortest prefix whose mass reaches thr
+    const uint64_t S = __reduce_add_sync(0xffffffffu, w);
+    const uint64_t prod = (uint64_t)p.p_fixed * S;
+    const uint64_t t = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
+    uint32_t incl = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    kept = kept && (lane == 0 || (uint64_t)(incl - w) < t);
+  }
+  const uint32_t kw = kept ? w : 0u;
+  const uint64_t Sk = __reduce_add_sync(0xffffffffu, kw);
+  const uint64_t tau = __umul64hi(rnd, Sk);
+  // ascending-id cumulative weight of the kept elements up to and including this lane's
+  uint64_t cum = 0;
+  for (int j = 0; j < nc; ++j) {
+    const uint32_t wj = __shfl_sync(0xffffffffu, kw, j);
+    const int idj = __shfl_sync(0xffffffffu, id, j);
+    if (idj <= id) cum += wj;
+  }
+  const uint32_t m = __ballot_sync(0xffffffffu, kept && cum > tau && cum - kw <= tau);
+  return __shfl_sync(0xffffffffu, id, __ffs(m) - 1);
+}
+
+// steps 4-7 of the sampler on the list (warp 0): candidates, kept set, draw, pick.  S_all is
+// the mass of every id (the candidates' mass when there is no top-k).
+__device__ int list_select(const AcceptParams& p, const NucList& L, int n, uint64_t S_all, uint64_t rnd) {
+  const int lane = threadIdx.x & 31;
+  // 4. top-k candidates: W > xk, or W == xk and id <= idk
+  uint32_t xk = 0;
+  int idk = 0x7FFFFFFF;
+  const bool topk = p.top_k > 0 && p.top_k < p.V;
+  if (topk && n >= p.top_k) {
+    const uint64_t k = (uint64_t)p.top_k;
+    xk = list_threshold<true>(L, n, k, [](uint32_t, int) { return true; });
+    const uint64_t above = list_sum<true>(L, n, [&](uint32_t w, int) { return w > xk; });
+    idk = list_nth(L, n, k - above, [&](uint32_t w, int) { return w == xk; });
+  }
+  // (n < k: the list holds every non-zero weight, all of them candidates; the zero-weight
+  // candidates add nothing to any sum and are never kept)
+  auto cand = [&](uint32_t w, int id) { return w > xk || (w == xk && id <= idk); };
+  // 5. top-p over the candidates
+  const uint64_t S = topk ? list_sum<false>(L, n, cand) : S_all;
+  const uint64_t prod = (uint64_t)p.p_fixed * S;
+  const uint64_t thr = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
+  uint32_t xp = 0;
+  int idp = -1;   // thr >= S: every non-zero candidate is kept
+  if (thr < S) {
+    xp = list_threshold<false>(L, n, thr, cand);
+    const uint64_t above = list_sum<false>(L, n, [&](uint32_t w, int id) { return cand(w, id) && w > xp; });
+    const uint64_t n_above = list_sum<true>(L, n, [&](uint32_t w, int id) { return cand(w, id) && w > xp; });
+    uint64_t ties = thr > above ? (thr - above + xp - 1) / xp : 0;
+    if (n_above == 0 && ties == 0) ties = 1;
+    idp = ties == 0 ? -1 : list_nth(L, n, ties, [&](uint32_t w, int id) { return cand(w, id) && w == xp; });
+  }
+  auto kept = [&](uint32_t w, int id) { return cand(w, id) && (w > xp || (w == xp && id <= idp)); };
+  const uint64_t Sk = list_sum<false>(L, n, kept);
+  // 6. the draw, 7. the first kept id whose inclusive cumulative weight exceeds tau
+  const uint64_t tau = __umul64hi(rnd, Sk);
+  uint64_t carry = 0;
+  for (int b = 0; b < n; b += 32) {
+    const int i = b + lane;
+    const uint32_t w = (i < n && kept(L.w[i], L.id[i])) ? L.w[i] : 0u;
+    uint32_t x = w;   // inclusive prefix within the chunk (< 2^29)
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    const uint32_t m = __ballot_sync(0xffffffffu, w != 0 && carry + x > tau);
+    if (m) return __shfl_sync(0xffffffffu, L.id[b + __ffs(m) - 1], 0);
+    carry += __shfl_sync(0xffffffffu, x, 31);
+  }
+  return 0x7FFFFFFF;   // not reached: tau < Sk
+}
+
 __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* row, int position, int seq,
-                                           float* redf, uint64_t* red, int* redi) {
+                                           float* redf, uint64_t* red, int* redi, NucList& L) {
   const int V = p.V;
   const int base = threadIdx.x * ACC_EPT;
   uint32_t W[ACC_EPT];
   float mx = -INFINITY;
   bool nan = false;
+  if (threadIdx.x < NUC_FLOORS) L.cnt[threadIdx.x] = 0;   // published by block_max_f's barriers
+  if (threadIdx.x < 3) L.mhi[threadIdx.x] = L.mlo[threadIdx.x] = 0;
   {
     // 1. logits (NaN -> -inf; ids >= V are -inf, hence W = 0) and the row maximum
     float l[ACC_EPT];
@@ -317,6 +511,103 @@ __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* r
 #pragma unroll
     for (int e = 0; e < ACC_EPT; ++e) W[e] = fixed24(exp_sd(__fdiv_rn(__fsub_rn(l[e], mx), p.temperature)));
   }
+  // 6. the 64-bit draw keyed by (produced position, sequence)
+  uint32_t ctr[4] = {(uint32_t)position, (uint32_t)seq, 0u, 0u};
+  philox4x32_10(ctr, (uint32_t)(p.seed & 0xFFFFFFFFull), (uint32_t)(p.seed >> 32));
+  const uint64_t rnd = ((uint64_t)ctr[0] << 32) | ctr[1];
+
+  // ---- the list path: counts (and, without top-k, masses) of the weights above each floor
+  {
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool topk = p.top_k > 0 && p.top_k < V;
+    uint32_t c01 = 0, c23 = 0, c45 = 0, c6 = 0;   // per-thread counts, two 11-bit fields per word
+    uint32_t m4 = 0, m5 = 0, m6 = 0;              // per-thread masses >= floors 4, 5, 6 (< 2^29)
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e) {
+      const int b = nuc_bucket(W[e]);
+      c01 += (b <= 0 ? 1u : 0u) + (b <= 1 ? 1u << 11 : 0u);
+      c23 += (b <= 2 ? 1u : 0u) + (b <= 3 ? 1u << 11 : 0u);
+      c45 += (b <= 4 ? 1u : 0u) + (b <= 5 ? 1u << 11 : 0u);
+      c6 += b <= 6 ? 1u : 0u;
+      if (!topk) {
+        m4 += b <= 4 ? W[e] : 0u;
+        m5 += b <= 5 ? W[e] : 0u;
+        m6 += W[e];
+      }
+    }
+    c01 = __reduce_add_sync(0xffffffffu, c01);   // warp totals <= 1024 per field
+    c23 = __reduce_add_sync(0xffffffffu, c23);
+    c45 = __reduce_add_sync(0xffffffffu, c45);
+    c6 = __reduce_add_sync(0xffffffffu, c6);
+    uint32_t mh[3] = {0, 0, 0}, ml[3] = {0, 0, 0};
+    if (!topk) {
+      const uint32_t m[3] = {m4, m5, m6};
+#pragma unroll
+      for (int i = 0; i < 3; ++i) {
+        mh[i] = __reduce_add_sync(0xffffffffu, m[i] >> 12);
+        ml[i] = __reduce_add_sync(0xffffffffu, m[i] & 4095u);
+      }
+    }
+    if (lane == 0) {
+      atomicAdd(&L.cnt[0], c01 & 2047u);
+      atomicAdd(&L.cnt[1], c01 >> 11);
+      atomicAdd(&L.cnt[2], c23 & 2047u);
+      atomicAdd(&L.cnt[3], c23 >> 11);
+      atomicAdd(&L.cnt[4], c45 & 2047u);
+      atomicAdd(&L.cnt[5], c45 >> 11);
+      atomicAdd(&L.cnt[6], c6);
+      if (!topk)
+#pragma unroll
+        for (int i = 0; i < 3; ++i) {
+          atomicAdd(&L.mhi[i], (unsigned long long)mh[i]);
+          atomicAdd(&L.mlo[i], (unsigned long long)ml[i]);
+        }
+    }
+    __syncthreads();
+    int N[NUC_FLOORS];
+#pragma unroll
+    for (int f = 0; f < NUC_FLOORS; ++f) N[f] = (int)L.cnt[f];
+    if (N[6] == 0) return 0;   // every weight 0 (all-NaN row): the lowest candidate, id 0
+    uint64_t Sf[3];
+#pragma unroll
+    for (int i = 0; i < 3; ++i) Sf[i] = (L.mhi[i] << 12) + L.mlo[i];
+    const uint64_t S_all = Sf[2];
+    uint64_t thr_all = 0;
+    if (!topk) {
+      const uint64_t prod = (uint64_t)p.p_fixed * S_all;
+      thr_all = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
+    }
+    // the highest floor whose elements provably hold the candidates (top-k) or the kept prefix
+    int f = -1;
+#pragma unroll
+    for (int i = 0; i < NUC_FLOORS; ++i) {
+      const bool holds = topk ? (N[i] >= p.top_k || N[i] == N[6]) : (i >= 4 && Sf[i - 4] >= thr_all);
+      if (f < 0 && N[i] <= NUC_LIST_MAX && holds) f = i;
+    }
+    if (f >= 0) {
+      uint32_t mine = 0;
+#pragma unroll
+      for (int e = 0; e < ACC_EPT; ++e) mine += nuc_bucket(W[e]) <= f;
+      uint32_t at = (uint32_t)block_exscan_u64(mine, red);
+#pragma unroll
+      for (int e = 0; e < ACC_EPT; ++e)
+        if (nuc_bucket(W[e]) <= f) {
+          L.w[at] = W[e];
+          L.id[at] = base + e;
+          ++at;
+        }
+      __syncthreads();
+      if (w == 0) {
+        int pick = list_small(p, L, N[f], S_all, topk, rnd);
+        if (pick < 0) pick = list_select(p, L, N[f], S_all, rnd);
+        if (lane == 0) L.pick = pick;
+      }
+      __syncthreads();
+      return L.pick;
+    }
+  }
+
+  // ---- the block-wide path over all ids
   Cut c;
   c.xk = 0;
   c.idk = 0x7FFFFFFF;
@@ -340,10 +631,6 @@ __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* r
   if (n_above == 0 && ties == 0) ties = 1;
   c.idp = ties == 0 ? -1 : nth_id<P_CAND_EQ>(W, base, c, c.xp, ties, red, redi);
   const uint64_t Sk = block_sum_u64(lsum<P_KEPT, false>(W, base, c, 0), red);
-  // 6. the 64-bit draw keyed by (produced position, sequence)
-  uint32_t ctr[4] = {(uint32_t)position, (uint32_t)seq, 0u, 0u};
-  philox4x32_10(ctr, (uint32_t)(p.seed & 0xFFFFFFFFull), (uint32_t)(p.seed >> 32));
-  const uint64_t rnd = ((uint64_t)ctr[0] << 32) | ctr[1];
   const uint64_t tau = __umul64hi(rnd, Sk);
   // 7. the first kept id (ascending) whose inclusive cumulative weight exceeds tau
   const uint64_t mine = lsum<P_KEPT, false>(W, base, c, 0);
@@ -390,6 +677,7 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
   __shared__ uint64_t red[32];
   __shared__ int redi[32];
   __shared__ int s_last;
+  __shared__ NucList nl;
   pdl_wait();
   pdl_trigger();
   const int j = blockIdx.x, sl = blockIdx.y, s = p.seq0 + sl;
@@ -400,7 +688,7 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
   } else {
     // the produced token's position: one past the row's own (len + j, or len + depth(j))
     const int position = __ldcg(p.len + s) + (p.parent ? tree_depth(p.parent + sl * p.q, j, nullptr) : j) + 1;
-    t = row_nucleus(p, row, position, s, redf, red, redi);
+    t = row_nucleus(p, row, position, s, redf, red, redi, nl);
   }
   if (threadIdx.x == 0) p.targets[sl * p.q + j] = t;
   __threadfence();

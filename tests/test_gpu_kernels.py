@@ -263,3 +263,42 @@ def test_accept_nucleus_full_vocab(sd):
         acc, out, flags, _ = _run_accept(ctx, lg, dr, b, q, q - 1, lens, T, p, 11, k)
         racc, rout = _oracle_accept(lgc, drafts, b, q, q - 1, lens, T, p, 11, k)
         assert out == rout and acc == racc
+
+
+def _nucleus_rows(V):
+    """Rows that steer the sampler's list path (heavy weights compacted, at each floor) and its
+    block-wide path (too many heavy weights), at the boundaries between them."""
+    rows = []
+    flat = torch.zeros(V)                                            # every weight 2^24: block-wide path
+    rows.append(flat)
+    peaked = torch.full((V,), -100.0)                                # three non-zero weights
+    peaked[[7, 300, 301]] = torch.tensor([0.0, -0.5, -0.5])
+    rows.append(peaked)
+    for n in (2048, 2049):                                           # list capacity, and one past it
+        r = torch.full((V,), -100.0)
+        r[torch.arange(n) * (V // n)] = 0.0
+        rows.append(r)
+    mid = torch.full((V,), -100.0)                                   # mass above 2^-8 of the max < 0.95
+    mid[5] = 0.0
+    mid[1000:1200] = -8.0
+    rows.append(mid)
+    g = torch.Generator().manual_seed(5)
+    rows.append(torch.randn(V, generator=g) * 0.3)                   # nearly flat
+    rows.append(torch.randn(V, generator=g) * 6.0)                   # peaked at T = 1
+    return torch.stack(rows).float()
+
+
+@pytest.mark.parametrize("T,top_p,top_k", [(1.0, 0.95, 0), (1.0, 0.95, 10), (0.2, 1.0, 0), (1.0, 0.5, 3),
+                                           (0.2, 0.95, 10), (1.0, 0.999, 0)])
+def test_accept_nucleus_list_and_block_paths(accept_env, T, top_p, top_k):
+    """Bit-exact against the oracle on rows built to take each of the sampler's paths."""
+    V = accept_env.shape.vocab
+    lg = _nucleus_rows(V)
+    n = lg.shape[0]
+    lgc = lg.numpy()
+    drafts = [0] * n
+    acc, out, flags, _ = _run_accept(accept_env, lg.cuda(), torch.zeros(n, dtype=torch.int32, device="cuda"), 1, n,
+                                     0, [40], T, top_p, 3, top_k)
+    _, rout = _oracle_accept(lgc, drafts, 1, n, 0, [40], T, top_p, 3, top_k)
+    assert out == rout
+    assert flags == 0
