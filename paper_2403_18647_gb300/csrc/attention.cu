@@ -450,11 +450,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
       if (p.trace.rec) t_part = globaltimer_ns();
       // the CTA's stores, then one release/acquire counter update by thread 0
       __syncthreads();
-      if (tid == 0) {
-        __threadfence();
-        *s_last = (atomicAdd(p.counters + sl * H + h, 1) == nseg - 1);
-        __threadfence();
-      }
+      if (tid == 0) *s_last = (atomic_add_acq_rel_gpu(p.counters + sl * H + h, 1) == nseg - 1);
       __syncthreads();
       if (*s_last && fits) {
         // ---- merge the pair's partials: w[j][s] = exp(m_s - max m), L_j = sum_s w[j][s] l_s,

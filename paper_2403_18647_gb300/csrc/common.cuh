@@ -129,6 +129,16 @@ __device__ __forceinline__ void bulk_load_g2s(void* dst, const void* src, uint32
 }
 // global-memory writes made visible through the generic proxy -> ordered before later
 // async-proxy (bulk copy) reads of the same locations
+// Split-K style publication: after a barrier orders the CTA's stores before it, one thread
+// adds to a counter with release semantics (cumulative over those stores) and acquire
+// semantics (the contributors that added before are visible to it, and through the next
+// barrier to the CTA), at GPU scope.
+__device__ __forceinline__ int atomic_add_acq_rel_gpu(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }

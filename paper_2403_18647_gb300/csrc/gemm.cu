@@ -477,11 +477,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
           if (m < p.M) mine[m * 128 + r] = acc[m];
         // publish: the CTA's stores, then one release/acquire counter update (thread r = 0)
         named_bar_sync(1, 128);
-        if (r == 0) {
-          __threadfence();
-          *s_last = (atomicAdd(&p.counters[tile], 1) == c_hi - c_lo);
-          __threadfence();
-        }
+        if (r == 0) *s_last = (atomic_add_acq_rel_gpu(&p.counters[tile], 1) == c_hi - c_lo);
         named_bar_sync(1, 128);
         if (r == 0 && last_seg && p.trace.rec) s_mark[3] = (unsigned long long)(*s_last) | ((c_hi - c_lo + 1) << 8);
         if (!*s_last) {
