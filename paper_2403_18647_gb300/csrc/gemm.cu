@@ -66,7 +66,9 @@ struct GemmCfg {
   static constexpr int ACC_COLS = 2 * MPAD;     // hi and lo products side by side
   static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
   static constexpr int NBAR = 2 * STAGES + 6;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + NBAR * 8 + 64;
+  static constexpr int CS = MPAD * 64;           // EPI_QKV: RoPE (cos, sin) of every row and frequency
+  static constexpr size_t SMEM =
+      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + CS * 8 + NBAR * 8 + 64;
 };
 
 __device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
@@ -100,7 +102,7 @@ template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
                                                float* staging, const float* sinv, const int* s_slot,
                                                const int* s_pos, const float (&pre)[EG], float pre_gn,
-                                               const float2 (&pre_cs)[EG]) {
+                                               const float2* s_cs) {
   const int M = p.M;
   if (p.ssq_in) {
 #pragma unroll
@@ -224,7 +226,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
           slot[u] = s_slot[m];
           val[u] = acc[m];
           if (which < 2) {   // rotate-half RoPE with the partner lane's value from shared memory
-            const float2 cs = m0 == 0 ? pre_cs[u] : p.rope[(size_t)s_pos[m] * half + (i % half)];
+            const float2 cs = s_cs[m * 64 + (i % half)];
             const float y = staging[partner * (MPAD + 1) + m];
             val[u] = (i < half) ? acc[m] * cs.x - y * cs.y : acc[m] * cs.x + y * cs.y;
           }
@@ -260,7 +262,8 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   float* sinv = staging + C::STAGING;   // [64] RMSNorm row factors of the operand
   int* s_slot = reinterpret_cast<int*>(sinv + 64);   // [64] EPI_QKV: cache slot of each row
   int* s_pos = s_slot + 64;                          // [64] EPI_QKV: RoPE position of each row
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_pos + 64);
+  float2* s_cs = reinterpret_cast<float2*>(s_pos + 64);   // [MPAD][64] EPI_QKV: RoPE factors
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_cs + C::CS);
   uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
   uint64_t* empty = bars + S;        // stage consumed by the tensor core
   uint64_t* acc_full = bars + 2 * S; // [2] accumulator ready
@@ -419,6 +422,11 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         s_pos[r] = pos;
       }
       named_bar_sync(1, 128);
+      // the RoPE factors of every row, in shared memory long before any accumulator is ready
+      const int half = max(p.hd >> 1, 1);
+      for (int i = r; i < p.M * half; i += 128)
+        s_cs[(i / half) * 64 + i % half] = p.rope[(size_t)s_pos[i / half] * half + i % half];
+      named_bar_sync(1, 128);
     }
     int seg = 0;
     long long g = g0;
@@ -427,21 +435,15 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
       g = std::min(g1, (long long)(tile + 1) * p.kc);
       const int buf = seg & 1;
       // what this tile's epilogue reads from global memory (first row group), loaded while
-      // the tensor cores work: residual rows and gain, or RoPE factors
+      // the tensor cores work: residual rows and gain
       float pre[EG];
       float pre_gn = 0.f;
-      float2 pre_cs[EG];
       {
         const int n = 128 * tile + r;
         const bool resid = p.epi == EPI_RESID && n < p.N;
 #pragma unroll
         for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
         if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
-        const bool rope = p.epi == EPI_QKV && n / p.rows_per_map < 2;   // a q or k feature (rows_per_map > 0)
-        const int half = max(p.hd >> 1, 1), ih = rope ? (n % p.rows_per_map) % p.hd % half : 0;
-#pragma unroll
-        for (int u = 0; u < EG; ++u)
-          pre_cs[u] = (rope && u < p.M) ? p.rope[(size_t)s_pos[u] * half + ih] : make_float2(1.f, 0.f);
       }
       const bool got = mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err);
       __syncwarp();   // lanes leave the polling loop at different times: reconverge
@@ -532,7 +534,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         if (r == 0) p.counters[tile] = 0;
       }
       if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
-      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn, pre_cs);
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn, s_cs);
     }
   }
 
