@@ -95,6 +95,16 @@ def peaks():
         return 6800.0, "fallback"
 
 
+def tensor_peak():
+    """Dense bf16 tensor-core peak (TFLOP/s): the measured burst cuBLAS figure, else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
 # ----------------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -198,6 +208,7 @@ class Runner:
         self.prompts = [synth.prompt_ids(0, s, self.P, self.shape.adaptive_id, device) for s in range(self.b)]
         for s in range(self.b):
             self.ctx.prefill(self.kv, s, self.prompts[s][:-1].contiguous())
+        self.prefill_ms = self._time_prefill()
         self.first = torch.stack([p[-1] for p in self.prompts]).to(torch.int32)
         # the loop starts as if a draft step 2 block (q2 rows) had just emitted the last prompt token
         self.init_out = torch.zeros_like(self.out)
@@ -207,6 +218,26 @@ class Runner:
         self.start_len = torch.full((self.b,), self.P - 1, dtype=torch.int32, device=device)
         self._make_table()
         torch.cuda.synchronize()
+
+    def _time_prefill(self, reps=3):
+        """Device time of sequence 0's prompt prefill (the step before the decode loop), rerun
+        from an empty cache after the first, untimed one."""
+        torch = self.torch
+        lens = self.ctx.kv_lengths(self.kv).clone()
+        zero = lens.clone()
+        zero[0] = 0
+        toks = self.prompts[0][:-1].contiguous()
+        times = []
+        for _ in range(reps):
+            self.ctx.kv_commit(self.kv, zero, self.b)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            self.ctx.prefill(self.kv, 0, toks)
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        self.ctx.kv_commit(self.kv, lens, self.b)
+        return min(times)
 
     # target selection for this workload
     def accept(self, n_verify, commit=True):
@@ -528,6 +559,7 @@ def run_ours(args, wl, rank, world):
         "kernels": {k: {"launches": v[0], "ms_total": round(v[1], 4), "us_per_launch": round(1e3 * v[1] / v[0], 2)}
                     for k, v in kstats.items()},
         "e2e": e2e, "gpu_launches": gpu_launches, "device_error_flags": flags,
+        "prefill": prefill_line(r),
     }
     if r.tree:
         out["config"].update({"tree_width": r.width, "q2": r.q2,
@@ -535,6 +567,23 @@ def run_ours(args, wl, rank, world):
     if clk:
         out["clocks"] = clk
     return r, out
+
+
+def prefill_line(r, chunk=512):
+    """The prompt prefill (not part of the timed decode steps): tokens/s and its tensor-core
+    rate.  FLOPs = 2 x positions x decoder-layer weights (the projections) + the causal
+    attention products 2 x 2 x n^2/2 x H x hd per layer (algorithmic; the hi + lo operand
+    split doubles what the tensor cores execute for the projections)."""
+    n = r.P - 1
+    sec = r.prefill_ms / 1e3
+    sh = r.shape
+    layer_w = sh.n_layers * (4 * sh.n_heads * sh.head_dim * sh.d_model + 3 * sh.ffn_dim * sh.d_model)
+    flops = 2.0 * n * layer_w + sh.n_layers * 2.0 * 2.0 * (n * n / 2.0) * sh.n_heads * sh.head_dim
+    tpk, kind = tensor_peak()
+    tf = flops / sec / 1e12
+    return {"tokens": n, "ms": round(r.prefill_ms, 3), "tokens_per_s": round(n / sec, 1), "chunk_rows": chunk,
+            "tflops": round(tf, 1), "frac_of_measured_bf16": round(tf / tpk, 4), "peak": tpk, "peak_source": kind,
+            "note": "tiled tcgen05 GEMM (128 weight rows x 128 positions), attention in 16-row causal groups"}
 
 
 def run_e2e(r, steps, steps_per_gen):
@@ -822,6 +871,34 @@ def run_sweep(args):
                               "frac_of_measured": round(by / us / 1e3 / peak, 4),
                               "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4)})
             del Ks, Vs
+    if args.sweep in ("prefill", "all"):
+        # the prefill path's tiled GEMM (M positions x the 7B projections), tensor-core bound
+        tpk, tkind = tensor_peak()
+        shapes = [tuple(int(v) for v in args.shape.split("x"))] if args.shape else SWEEP_GEMM_SHAPES[:3]
+        ms = [args.m] if args.m else [128, 256, 512]
+        for K, N in shapes:
+            w = synth.normal_bf16(9, 1, (N, K), 0.02, device="cuda")
+            for M in ms:
+                x = synth.normal_f32(9, 100 + M, (M, K), 1.0, device="cuda")
+                y = torch.empty(M, N, device="cuda")
+                for i in range(3):
+                    ctx.op_gemm(x, w, y)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                for i in range(reps):
+                    ctx.op_gemm(x, w, y)
+                e1.record()
+                torch.cuda.synchronize()
+                us = e0.elapsed_time(e1) * 1e3 / reps
+                alg = 2.0 * M * N * K / us / 1e6          # TFLOP/s of y = x W^T
+                cases.append({"kernel": "prefill_gemm", "M": M, "K": K, "N": N, "us": round(us, 2),
+                              "TFLOP/s": round(alg, 1), "frac_of_measured_bf16": round(alg / tpk, 4),
+                              "tensor_TFLOP/s": round(2 * alg, 1), "tensor_frac": round(2 * alg / tpk, 4),
+                              "peak": tpk, "peak_source": tkind,
+                              "note": "x enters as bf16 hi + lo: the tensor cores execute 2 x 2MNK; includes "
+                                      "the fp32 -> bf16 hi/lo operand split kernel"})
+            del w
     for c in cases:
         print(json.dumps(c), flush=True)
 
@@ -834,7 +911,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="7b", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--sweep", choices=["gemm", "attention", "all"], help="kernel sweeps instead of the step bench")
+    ap.add_argument("--sweep", choices=["gemm", "attention", "prefill", "all"],
+                    help="kernel sweeps instead of the step bench")
     ap.add_argument("--shape", default="", help="sweep one GEMM shape KxN")
     ap.add_argument("--m", type=int, default=0, help="sweep one M (GEMM) or q (attention)")
     ap.add_argument("--ctx", type=int, default=0, help="sweep one attention context length")

@@ -287,9 +287,13 @@ SDSAT_API sdsat_status sdsat_build_tree_block(sdsat_ctx* ctx, sdsat_kv* kv, int 
                                               const int32_t* draft_tables_dev, int width, int table_stride, int b,
                                               int k, int32_t* tokens_out_dev);
 
-/* Run n prompt tokens of sequence `seq` through the model in blocks of up to
- * SDSAT_MAX_Q rows and commit them (len[seq] += n).  No logits are produced.
- * Errors: EINVAL. */
+/* Run n prompt tokens of sequence `seq` through the model and commit them
+ * (len[seq] += n): the step before the decode loop.  Chunks of up to
+ * SDSAT_MAX_ROWS positions go through one block forward each (the weights stream
+ * once per chunk), position i attending to every earlier position; a tail shorter
+ * than SDSAT_MAX_Q rows runs as one ordinary block.  No logits are produced.
+ * Errors: EINVAL (null pointer, seq outside the KV batch, n < 0), ECAPACITY
+ * (n > max_len); device bit CAPACITY if len[seq] + n > max_len. */
 SDSAT_API sdsat_status sdsat_prefill(sdsat_ctx* ctx, sdsat_kv* kv, int seq, const int32_t* tokens_dev, int n);
 
 /* Synchronise the context stream, return the accumulated device error bits in
@@ -301,9 +305,12 @@ SDSAT_API const char* sdsat_status_string(sdsat_status s);
 
 /* ---- single kernels (unit parity tests and kernel sweeps) ------------------------- */
 
-/* y[m][n] = sum_k x[m][k] * W[n][k] for m < M, n < N: the weight-streaming skinny
- * GEMM behind every projection of the block forward.  x fp32 [M][K] (row stride
- * K), W bf16 [N][K], y fp32 [M][N].  M <= SDSAT_MAX_ROWS.  Errors: EINVAL. */
+/* y[m][n] = sum_k x[m][k] * W[n][k] for m < M, n < N.  M <= SDSAT_MAX_ROWS runs the
+ * weight-streaming skinny GEMM behind every projection of the block forward;
+ * SDSAT_MAX_ROWS < M <= 512 runs the tiled GEMM of the prefill path (128 weight rows
+ * x 128 positions per tile).  x fp32
+ * [M][K] (row stride K), W bf16 [N][K], y fp32 [M][N]; x and W 16-byte aligned,
+ * K a multiple of 8, K <= 32768.  Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_op_gemm(sdsat_ctx* ctx, const float* x_dev, int M, int K, const void* w_dev, int N,
                            float* y_dev);
 

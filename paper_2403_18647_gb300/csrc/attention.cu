@@ -4,7 +4,9 @@
 // [0, len[s]) and to block rows 0..j (slots len[s] .. len[s]+j), which the QKV
 // epilogue has just written; this is how Eq. 1-2 evaluate every appended
 // position of the block in one pass.  A tree block (Sec. 2.1.2) replaces the
-// rows 0..j by row j's ancestors and itself, given as one bit mask per row.
+// rows 0..j by row j's ancestors and itself, given as one bit mask per row.  A
+// prefill chunk of one sequence runs as consecutive groups of q rows: group g
+// sees len + g*q committed slots, then its rows causally.
 // The bytes are the K and V rows (bf16, hd*2 bytes each), read once per
 // (sequence, head) for all q rows together.
 //
@@ -124,7 +126,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   // first kernel (RMSNorm) lets its dependents launch only after every earlier kernel
   // has completed.  Slots below them are not written during this forward either.
   if (tid < p.nb) {
-    const int len = __ldcg(p.len + p.seq0 + tid);
+    const int len = p.groups ? __ldcg(p.len + p.seq0) + tid * q : __ldcg(p.len + p.seq0 + tid);
     len_seq[tid] = len;
     nu_seq[tid] = (min(len + q, p.cap) + ATT_UNIT - 1) / ATT_UNIT;
   }
@@ -162,8 +164,10 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   auto unit_row = [&](int u, bool& committed) {
     int s, hh, cc;
     locate(u, s, hh, cc);
-    committed = (cc + 1) * ATT_UNIT <= len_seq[s];
-    return p.row0 + ((p.seq0 + s) * H + hh) * p.cap + cc * ATT_UNIT;
+    // (prefill groups: the slots after the sequence's committed length are this chunk's rows,
+    // written by the kernel before)
+    committed = (cc + 1) * ATT_UNIT <= (p.groups ? len_seq[0] : len_seq[s]);
+    return p.row0 + ((p.seq0 + (p.groups ? 0 : s)) * H + hh) * p.cap + cc * ATT_UNIT;
   };
   uint64_t pol = 0;
   auto issue = [&](int k, int row) {   // unit u0 + k into stage k % ATT_STAGES

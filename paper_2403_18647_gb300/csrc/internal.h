@@ -119,6 +119,8 @@ struct AttnParams {
   const int* len;       // [B]
   const uint32_t* anc;  // [nb*q] tree blocks: bit i of row j = row j attends block row i; null = causal
   int seq0, nb, q, H, hd, cap;
+  int groups;           // prefill: the nb "sequences" are consecutive groups of q rows of sequence
+                        //   seq0 (group g sees len[seq0] + g*q committed slots, then causal)
   float* out;           // [rows][out_ld] fp32
   int out_ld;
   __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
@@ -133,6 +135,38 @@ size_t attention_smem_bytes(int hd);
 cudaError_t attention_prepare();   // set smem attributes (idempotent)
 // grid: min(2 * num_sms, 14 * H) CTAs, so at most ATT_SEG_MAX CTAs share one (sequence, head)
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl);
+
+// ---- prefill (prompt chunks of up to PF_ROWS positions) -------------------------
+constexpr int PF_ROWS = 512;
+struct PfGemmParams {
+  CUtensorMap tmap[3];      // weights, as GemmParams::tmap (map_mode)
+  CUtensorMap tmap_x[2];    // positions' operand, bf16 hi / lo [PF_ROWS][K], boxes of 64 x 128
+  int map_mode, rows_per_map;
+  int N;                    // output features (MAP_GATEUP: F)
+  int kc;                   // 64-column chunks of K
+  int n_wtiles, n_tblocks;  // tiles of 128 weight rows, blocks of 128 positions
+  int M;                    // positions
+  int epi;                  // EPI_STORE, EPI_RESID or EPI_SWIGLU
+  float* out;               // [M][out_ld] fp32 (EPI_STORE, EPI_RESID)
+  int out_ld;
+  __nv_bfloat16* out_hi;    // EPI_SWIGLU: [M][out_ld] the down projection's operand
+  __nv_bfloat16* out_lo;
+  uint32_t* err;
+};
+cudaError_t prefill_prepare();
+cudaError_t launch_prefill_gemm(PfGemmParams& p, int num_sms, cudaStream_t st, bool pdl);
+struct RopeKvParams {
+  const float* qkv;         // [M][3R]
+  float* qout;              // [M][R]
+  __nv_bfloat16* k_layer;   // this layer's caches [B][H][cap][hd]
+  __nv_bfloat16* v_layer;
+  const int* len;
+  int seq, H, hd, cap;
+  const float2* rope;
+  int rope_len;
+  uint32_t* err;
+};
+cudaError_t launch_rope_kv(const RopeKvParams& p, int M, cudaStream_t st, bool pdl);
 
 // ---- embedding, acceptance, block building ------------------------------------
 // x = h * rsqrt(mean h^2 + eps) * g, stored as bf16 hi + lo (tokens != null: h = E[tokens] first)

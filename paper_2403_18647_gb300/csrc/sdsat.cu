@@ -87,11 +87,13 @@ struct LayerMaps {
 // kernel classes for the profiling hook
 enum KClass : int {
   K_RMSNORM = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
-  K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_TREE_PREP, K_TREE_COMPACT, K_COUNT
+  K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_TREE_PREP, K_TREE_COMPACT,
+  K_PF_GEMM, K_PF_ROPE_KV, K_COUNT
 };
 const char* const KCLASS_NAME[K_COUNT] = {"rmsnorm", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
                                           "gemm_lm_head", "accept", "build_block", "kv_commit", "prefill_commit",
-                                          "gemm_op", "attention_op", "tree_prep", "tree_compact"};
+                                          "gemm_op", "attention_op", "tree_prep", "tree_compact", "prefill_gemm",
+                                          "prefill_rope_kv"};
 
 constexpr int MAX_GEMM_TILES = 1 << 16;
 constexpr int OP_MAX_K = 32768;   // K limit of sdsat_op_gemm (its operand scratch is sized at create)
@@ -131,6 +133,17 @@ struct sdsat_ctx {
   int* tree_ws = nullptr;      // [SDSAT_MAX_ROWS][TREE_WS_STRIDE] tree commit: len, m, path
   int* adaptive = nullptr;
   uint32_t* err = nullptr;
+  // prefill workspaces (chunks of up to PF_ROWS positions; allocated with the weights)
+  float* pf_h = nullptr;         // [PF_ROWS][d] residual stream
+  float* pf_qkv = nullptr;       // [PF_ROWS][3R] projections before RoPE
+  float* pf_q = nullptr;         // [PF_ROWS][R] rotated queries
+  float* pf_attn = nullptr;      // [PF_ROWS][R] attention output
+  float* pf_part_o = nullptr;    // attention partials for PF_ROWS rows
+  float* pf_part_ml = nullptr;
+  int* pf_att_counters = nullptr;
+  __nv_bfloat16* pf_hi[X_COUNT] = {};   // GEMM operands [PF_ROWS][K] (normed x, attention, act)
+  __nv_bfloat16* pf_lo[X_COUNT] = {};
+  CUtensorMap pf_xmap[X_COUNT][2];      // boxes of 64 x 128
   __nv_bfloat16* x_hi[X_COUNT] = {};
   __nv_bfloat16* x_lo[X_COUNT] = {};
   CUtensorMap xmap[X_COUNT][3][2];     // [source][MPAD 16/32/64][hi/lo]
@@ -393,6 +406,118 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
   return SDSAT_OK;
 }
 
+// one prefill chunk: M (a multiple of SDSAT_MAX_Q, <= PF_ROWS) prompt positions of sequence seq
+// through every layer on the tiled GEMM, then committed
+sdsat_status prefill_chunk(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* tokens, int M) {
+  const sdsat_config& cf = c->cfg;
+  const int d = cf.d_model, H = cf.n_heads, hd = cf.head_dim, F = cf.ffn_dim, R = H * hd, L = cf.n_layers;
+  cudaStream_t st = c->stream;
+  const size_t layer_elems = (size_t)kv->batch * H * kv->cap * hd;
+  const int ntb = (M + 127) / 128;
+  auto norm = [&](const int32_t* toks, const void* gain) {
+    return timed(c, K_RMSNORM, [&] {
+      return launch_rmsnorm(toks, static_cast<const __nv_bfloat16*>(c->w.embed), cf.vocab, c->pf_h, d, M,
+                            static_cast<const __nv_bfloat16*>(gain), cf.rms_eps, c->pf_hi[X_NORM], c->pf_lo[X_NORM],
+                            c->err, st, c->pdl);
+    });
+  };
+  auto base = [&](int xsrc, int K) {
+    PfGemmParams g;
+    std::memset(&g, 0, sizeof(g));
+    g.tmap_x[0] = c->pf_xmap[xsrc][0];
+    g.tmap_x[1] = c->pf_xmap[xsrc][1];
+    g.kc = (K + 63) / 64;
+    g.n_tblocks = ntb;
+    g.M = M;
+    g.err = c->err;
+    return g;
+  };
+  auto gemm = [&](PfGemmParams& g) {
+    return timed(c, K_PF_GEMM, [&] { return launch_prefill_gemm(g, c->num_sms, st, c->pdl); });
+  };
+  if (norm(tokens, c->layers[0].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
+  for (int l = 0; l < L; ++l) {
+    const LayerMaps& mp = c->maps[l];
+    PfGemmParams gq = base(X_NORM, d);
+    gq.tmap[0] = mp.q;
+    gq.tmap[1] = mp.k;
+    gq.tmap[2] = mp.v;
+    gq.map_mode = MAP_QKV3;
+    gq.rows_per_map = R;
+    gq.N = 3 * R;
+    gq.n_wtiles = 3 * R / 128;
+    gq.epi = EPI_STORE;
+    gq.out = c->pf_qkv;
+    gq.out_ld = 3 * R;
+    if (gemm(gq) != cudaSuccess) return SDSAT_ECUDA;
+    RopeKvParams rp{c->pf_qkv, c->pf_q, kv->k + l * layer_elems, kv->v + l * layer_elems, kv->len, seq, H, hd,
+                    kv->cap, c->rope, cf.max_position, c->err};
+    if (timed(c, K_PF_ROPE_KV, [&] { return launch_rope_kv(rp, M, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
+    // attention: the chunk as causal groups of SDSAT_MAX_Q positions over the cache
+    AttnParams a;
+    std::memset(&a, 0, sizeof(a));
+    a.kmap = kv->kmap;
+    a.vmap = kv->vmap;
+    a.row0 = l * kv->batch * H * kv->cap;
+    a.Q = c->pf_q;
+    a.q_ld = R;
+    a.len = kv->len;
+    a.groups = 1;
+    a.seq0 = seq;
+    a.nb = M / SDSAT_MAX_Q;
+    a.q = SDSAT_MAX_Q;
+    a.H = H;
+    a.hd = hd;
+    a.cap = kv->cap;
+    a.out = c->pf_attn;
+    a.out_ld = R;
+    a.out_hi = c->pf_hi[X_ATTN];
+    a.out_lo = c->pf_lo[X_ATTN];
+    a.part_o = c->pf_part_o;
+    a.part_ml = c->pf_part_ml;
+    a.counters = c->pf_att_counters;
+    a.err = c->err;
+    a.trace = next_trace(c, K_ATTENTION);
+    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, c->num_sms, st, c->pdl); }) != cudaSuccess)
+      return SDSAT_ECUDA;
+    PfGemmParams go = base(X_ATTN, R);
+    go.tmap[0] = mp.o;
+    go.map_mode = MAP_PLAIN;
+    go.N = d;
+    go.n_wtiles = (d + 127) / 128;
+    go.epi = EPI_RESID;
+    go.out = c->pf_h;
+    go.out_ld = d;
+    if (gemm(go) != cudaSuccess) return SDSAT_ECUDA;
+    if (norm(nullptr, c->layers[l].ffn_norm) != cudaSuccess) return SDSAT_ECUDA;
+    PfGemmParams gg = base(X_NORM, d);
+    gg.tmap[0] = mp.gate;
+    gg.tmap[1] = mp.up;
+    gg.map_mode = MAP_GATEUP;
+    gg.N = F;
+    gg.n_wtiles = (F + 63) / 64;
+    gg.epi = EPI_SWIGLU;
+    gg.out_hi = c->pf_hi[X_FFN];
+    gg.out_lo = c->pf_lo[X_FFN];
+    gg.out_ld = F;
+    if (gemm(gg) != cudaSuccess) return SDSAT_ECUDA;
+    PfGemmParams gd = base(X_FFN, F);
+    gd.tmap[0] = mp.down;
+    gd.map_mode = MAP_PLAIN;
+    gd.N = d;
+    gd.n_wtiles = (d + 127) / 128;
+    gd.epi = EPI_RESID;
+    gd.out = c->pf_h;
+    gd.out_ld = d;
+    if (gemm(gd) != cudaSuccess) return SDSAT_ECUDA;
+    if (l + 1 < L && norm(nullptr, c->layers[l + 1].attn_norm) != cudaSuccess) return SDSAT_ECUDA;
+  }
+  return timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, M, kv->cap, c->err, st, c->pdl); }) ==
+                 cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
+}
+
 sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, const int32_t* drafts, int b, int q,
                            int n_verify, float top_p, float temperature, uint64_t seed, int top_k, int32_t* acc,
                            int32_t* out, int commit, const int32_t* parent = nullptr, int32_t* path = nullptr) {
@@ -481,7 +606,7 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
   }
   if (cudaGetDevice(&c->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess ||
-      gemm_prepare() != cudaSuccess || attention_prepare() != cudaSuccess) {
+      gemm_prepare() != cudaSuccess || attention_prepare() != cudaSuccess || prefill_prepare() != cudaSuccess) {
     delete c;
     return SDSAT_ECUDA;
   }
@@ -536,15 +661,26 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
             dalloc(c, &c->tree_pos, rows) && dalloc(c, &c->tree_anc, rows) &&
             dalloc(c, &c->tree_ws, (size_t)rows * TREE_WS_STRIDE) &&
-            dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)rows * OP_MAX_K) &&
+            dalloc(c, &c->err, 1) && dalloc(c, &c->xop_hi, (size_t)PF_ROWS * OP_MAX_K) &&
             dalloc(c, &c->ssq, (size_t)rows * ((d + 127) / 128)) &&
-            dalloc(c, &c->xop_lo, (size_t)rows * OP_MAX_K);
+            dalloc(c, &c->xop_lo, (size_t)PF_ROWS * OP_MAX_K);
   const int xcols[X_COUNT] = {d, R, F};
   for (int xs = 0; ok && xs < X_COUNT; ++xs) {
     ok = dalloc(c, &c->x_hi[xs], (size_t)rows * xcols[xs]) && dalloc(c, &c->x_lo[xs], (size_t)rows * xcols[xs]);
     for (int mi = 0; ok && mi < 3; ++mi)
       ok = make_xmap(&c->xmap[xs][mi][0], c->x_hi[xs], rows, xcols[xs], 16 << mi) &&
            make_xmap(&c->xmap[xs][mi][1], c->x_lo[xs], rows, xcols[xs], 16 << mi);
+  }
+  if (ok && c->has_weights) {
+    const int pr = PF_ROWS, H = cfg->n_heads, hd = cfg->head_dim;
+    ok = dalloc(c, &c->pf_h, (size_t)pr * d) && dalloc(c, &c->pf_qkv, (size_t)pr * 3 * R) &&
+         dalloc(c, &c->pf_q, (size_t)pr * R) && dalloc(c, &c->pf_attn, (size_t)pr * R) &&
+         dalloc(c, &c->pf_part_o, (size_t)pr * H * ATT_SEG_MAX * hd) &&
+         dalloc(c, &c->pf_part_ml, (size_t)pr * H * ATT_SEG_MAX * 2) && dalloc(c, &c->pf_att_counters, (size_t)pr * H);
+    for (int xs = 0; ok && xs < X_COUNT; ++xs)
+      ok = dalloc(c, &c->pf_hi[xs], (size_t)pr * xcols[xs]) && dalloc(c, &c->pf_lo[xs], (size_t)pr * xcols[xs]) &&
+           make_xmap(&c->pf_xmap[xs][0], c->pf_hi[xs], pr, xcols[xs], 128) &&
+           make_xmap(&c->pf_xmap[xs][1], c->pf_lo[xs], pr, xcols[xs], 128);
   }
   if (!ok) {
     sdsat_destroy(c);
@@ -697,13 +833,23 @@ sdsat_status sdsat_prefill(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
   if (!c || !kv || kv->ctx != c || !c->has_weights || !tokens_dev || seq < 0 || seq >= kv->batch || n < 0)
     return SDSAT_EINVAL;
   if (n > kv->cap) return SDSAT_ECAPACITY;
-  for (int i = 0; i < n; i += SDSAT_MAX_Q) {
-    const int qn = std::min(SDSAT_MAX_Q, n - i);
-    const sdsat_status s = forward(c, kv, seq, 1, qn, tokens_dev + i, nullptr, nullptr);
+  // chunks of up to PF_ROWS positions (a multiple of SDSAT_MAX_Q) on the tiled GEMM; a tail
+  // shorter than SDSAT_MAX_Q runs as one ordinary block
+  for (int i = 0; i < n;) {
+    const int rem = n - i;
+    if (rem >= SDSAT_MAX_Q) {
+      const int M = std::min(PF_ROWS, rem / SDSAT_MAX_Q * SDSAT_MAX_Q);
+      const sdsat_status s = prefill_chunk(c, kv, seq, tokens_dev + i, M);
+      if (s != SDSAT_OK) return s;
+      i += M;
+      continue;
+    }
+    const sdsat_status s = forward(c, kv, seq, 1, rem, tokens_dev + i, nullptr, nullptr);
     if (s != SDSAT_OK) return s;
-    if (timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, qn, kv->cap, c->err, c->stream, c->pdl); }) !=
+    if (timed(c, K_PREFILL_COMMIT, [&] { return launch_add_len(kv->len, seq, rem, kv->cap, c->err, c->stream, c->pdl); }) !=
         cudaSuccess)
       return SDSAT_ECUDA;
+    i += rem;
   }
   return SDSAT_OK;
 }
@@ -882,8 +1028,31 @@ sdsat_status sdsat_get_error(sdsat_ctx* c, uint32_t* flags) {
 
 sdsat_status sdsat_op_gemm(sdsat_ctx* c, const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev) {
   if (!c || !x_dev || !y_dev || !aligned16(w_dev) || !aligned16(x_dev)) return SDSAT_EINVAL;
-  if (M < 1 || M > SDSAT_MAX_ROWS || K < 8 || K % 8 || K > OP_MAX_K || N < 1 || (N + 127) / 128 > MAX_GEMM_TILES)
+  if (M < 1 || M > PF_ROWS || K < 8 || K % 8 || K > OP_MAX_K || N < 1 || (N + 127) / 128 > MAX_GEMM_TILES)
     return SDSAT_EINVAL;
+  if (M > SDSAT_MAX_ROWS) {
+    // the prefill GEMM (tiles of 128 weight rows x 128 positions)
+    const int rows = (M + 127) / 128 * 128;   // <= PF_ROWS rows of the operand scratch
+    PfGemmParams g;
+    std::memset(&g, 0, sizeof(g));
+    if (!make_wmap(&g.tmap[0], w_dev, N, K) || !make_xmap(&g.tmap_x[0], c->xop_hi, rows, K, 128) ||
+        !make_xmap(&g.tmap_x[1], c->xop_lo, rows, K, 128))
+      return SDSAT_ECUDA;
+    g.map_mode = MAP_PLAIN;
+    g.N = N;
+    g.kc = (K + 63) / 64;
+    g.n_wtiles = (N + 127) / 128;
+    g.n_tblocks = rows / 128;
+    g.M = M;
+    g.epi = EPI_STORE;
+    g.out = y_dev;
+    g.out_ld = N;
+    g.err = c->err;
+    if (launch_split(x_dev, M, K, c->xop_hi, c->xop_lo, c->stream, c->pdl) != cudaSuccess) return SDSAT_ECUDA;
+    return timed(c, K_GEMM_OP, [&] { return launch_prefill_gemm(g, c->num_sms, c->stream, c->pdl); }) == cudaSuccess
+               ? SDSAT_OK
+               : SDSAT_ECUDA;
+  }
   GemmParams g = gemm_base(c, M, -1);
   CUtensorMap m;
   if (!make_wmap(&m, w_dev, N, K) || !make_xmap(&g.tmap_x[0], c->xop_hi, SDSAT_MAX_ROWS, K, 16 << mpad_index(M)) ||

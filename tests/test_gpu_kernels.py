@@ -58,6 +58,8 @@ GEMM_CASES = [
     # (M, K, N): tiles, ragged N tail, ragged K tail (688 = 10.75 chunks), split-K sharing
     (1, 256, 256), (6, 256, 768), (6, 688, 256), (16, 256, 4104), (17, 512, 300), (24, 256, 1376),
     (33, 128, 130), (64, 256, 512), (6, 4096, 384), (2, 11008, 256),
+    # the tiled prefill GEMM: partial position blocks, ragged N and K, several waves of tiles
+    (65, 256, 256), (128, 688, 300), (200, 1024, 1000), (512, 4096, 384), (300, 512, 5000),
 ]
 
 
