@@ -14,6 +14,12 @@ sampling  argmax with the lowest-id tie break, the fixed-point nucleus
           (top-p) sampler, the exp used by it, and Philox4x32-10.
 decode    Eq. 3 verification, the two-step-draft-then-verify loops (greedy,
           and chain-form nucleus, Sec. 2.1.2) and plain decoding loops.
+tree      the tree-structured draft step 2 (Sec. 2.1.2): tree forward with
+          depth positions and ancestor masks, longest accepted branch, KV
+          compaction, the tree decoding loop.
+pipelined the pipelined variant (not a step of the paper): the verification
+          block also carries the adaptive tokens, so a loop whose drafts are
+          all accepted needs no separate draft step 1.
 
 Pins (tests/test_oracle_*.py) tie every function to something other than
 itself: closed forms, invariants the method fixes (greedy SDSAT output equals
