@@ -48,6 +48,11 @@ WORKLOADS = {
     # nucleus setting), k = 5 = tree depth, two chains of drafts below the root (q = 11)
     "7b-tree": dict(shape="7b", batch=1, prompt=2048, new=256, k=5, temperature=0.2, top_p=0.95, top_k=10,
                     match=0.6, width=2, match2=0.4),
+    # 7B shape, greedy, the pipelined variant (not a step of the paper): every block carries
+    # y, the k drafts and the k adaptive tokens (q = 2k + 1); a fully accepted block skips
+    # the next draft step 1
+    "7b-pipelined": dict(shape="7b", batch=1, prompt=2048, new=256, k=5, temperature=0.0, top_p=1.0, top_k=0,
+                         match=0.7, pipelined=True),
     # tiny correctness shape
     "tiny": dict(shape="tiny", batch=1, prompt=128, new=64, k=5, temperature=0.0, top_p=1.0, top_k=0, match=0.7),
 }
@@ -74,6 +79,15 @@ def expected_tokens_per_step(k: int, match: float, matches=None) -> float:
             miss *= 1.0 - p ** i
         tail += 1.0 - miss
     return (2.0 + tail) / 2.0
+
+
+def expected_tokens_per_step_pipelined(k: int, match: float) -> float:
+    """Pipelined blocks (stub coins with rate `match`): a mode-A block emits 1 + m and stays
+    in mode A iff m = k (probability p^k), a mode-S block emits 1 and leads to mode A;
+    stationary mean tokens per block."""
+    pk = match ** k
+    pi_a = 1.0 / (2.0 - pk)
+    return pi_a * (1.0 + sum(match ** i for i in range(1, k + 1))) + (1.0 - pi_a)
 
 
 def branch_matches(wl):
@@ -187,10 +201,12 @@ class Runner:
         self.wl = wl
         self.shape = synth.SHAPES[wl["shape"]]
         self.b, self.k = wl["batch"], wl["k"]
-        self.q = self.k + 1                       # draft step 1 block rows
+        self.pipe = bool(wl.get("pipelined"))
+        self.kinds = 1 if self.pipe else 2        # step kinds of a loop (graphs)
+        self.q = 2 * self.k + 1 if self.pipe else self.k + 1   # draft step 1 block rows (pipelined: every block)
         self.width = wl.get("width", 1)
         self.tree = self.width > 1
-        self.q2 = 1 + self.width * self.k         # draft step 2 block rows (the tree; the chain: q)
+        self.q2 = self.q if self.pipe else 1 + self.width * self.k   # draft step 2 block rows (chain: q)
         self.qmax = max(self.q, self.q2)
         self.P = wl["prompt"]
         self.new = wl["new"]
@@ -206,6 +222,8 @@ class Runner:
         self.acc = torch.ones(self.b, dtype=torch.int32, device=device)
         self.out = torch.zeros(self.b * self.qmax, dtype=torch.int32, device=device)
         self.parent = torch.tensor(chains_parent(self.width, self.k) * self.b, dtype=torch.int32, device=device)
+        self.pmode = torch.ones(self.b, dtype=torch.int32, device=device)    # pipelined: the previous block's mode
+        self.pnver = torch.zeros(self.b, dtype=torch.int32, device=device)
         self.prompts = [synth.prompt_ids(0, s, self.P, self.shape.adaptive_id, device) for s in range(self.b)]
         for s in range(self.b):
             self.ctx.prefill(self.kv, s, self.prompts[s][:-1].contiguous())
@@ -285,8 +303,17 @@ class Runner:
         self.ctx.kv_commit(self.kv, self.start_len, self.b)
         self.out.copy_(self.init_out)
         self.acc.copy_(self.init_acc)
+        self.pmode.fill_(1)
 
     def step(self, mode):
+        if self.pipe:
+            wl = self.wl
+            self.ctx.build_pipelined_block(self.kv, self.out, self.acc, self.pmode, self.pnver, self.toks, self.b,
+                                           self.k, draft_table=self.table, table_stride=self.stride)
+            self.ctx.block_forward(self.kv, self.toks, self.logits, self.b, self.q)
+            self.ctx.accept_pipelined(self.kv, self.logits, self.toks, self.pnver, self.b, self.q, self.acc, self.out,
+                                      temperature=wl["temperature"], top_p=wl["top_p"], seed=1234, top_k=wl["top_k"])
+            return
         if not self.tree:
             self.ctx.build_block(self.kv, mode, self.out, self.acc, self.toks, self.b, self.q,
                                  draft_table=self.table if mode == 2 else None, table_stride=self.stride)
@@ -323,7 +350,7 @@ class Runner:
             n += 1
             em = (self.ctx.kv_emitted(self.kv) - base).cpu().tolist()
             toks.append(sum(em) - sum(toks))
-            if n % 2 == 0 and min(em) >= self.new:
+            if n % self.kinds == 0 and min(em) >= self.new:
                 break
         flags = self.ctx.get_error()
         return n, lens, toks, flags
@@ -335,11 +362,11 @@ class Runner:
             s = torch.cuda.Stream()
             s.wait_stream(torch.cuda.current_stream())
             with torch.cuda.stream(s):
-                for mode in (1, 2):           # warm the path on the capture stream
+                for mode in (1, 2)[:self.kinds]:   # warm the path on the capture stream
                     self.step(mode)
             torch.cuda.current_stream().wait_stream(s)
             torch.cuda.synchronize()
-            for mode in (1, 2):
+            for mode in (1, 2)[:self.kinds]:
                 g = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g):
                     self.step(mode)
@@ -360,9 +387,9 @@ class Runner:
         for i in range(start, start + n):
             j = i % steps_per_gen
             if j == 0 and i > 0:
-                graphs[2].replay() if graphs else self.reset()
+                graphs[self.kinds].replay() if graphs else self.reset()
             if graphs:
-                graphs[j % 2].replay()
+                graphs[j % self.kinds].replay()
             else:
                 self.step(1 if j % 2 == 0 else 2)
 
@@ -370,6 +397,8 @@ class Runner:
 def accept_rate(r, toks):
     """Mean fraction of the k drafts accepted per verify step (draft step 2), from one
     calibrated generation: a verify step emits 1 + m tokens per sequence."""
+    if r.pipe:   # every block: the mean fraction of k accepted over the blocks that verified
+        return None
     ver = [t for i, t in enumerate(toks) if i % 2 == 1]
     if not ver:
         return None
@@ -388,8 +417,8 @@ def step_latency(r, graphs, steps_per_gen, n):
     for i in range(n):
         j = i % steps_per_gen
         if j == 0 and i > 0:
-            graphs[2].replay()
-        graphs[j % 2].replay()
+            graphs[r.kinds].replay()
+        graphs[j % r.kinds].replay()
         ev[i + 1].record()
     torch.cuda.synchronize()
     t = sorted(ev[i].elapsed_time(ev[i + 1]) for i in range(n))
@@ -545,7 +574,8 @@ def run_ours(args, wl, rank, world):
         "step_latency_ms": lat,
         "plain_decoding": plain,
         "speedup_vs_plain": round(value / world / plain["tokens_per_s"], 3) if plain else None,
-        "expected_tokens_per_step": round(expected_tokens_per_step(r.k, wl["match"], branch_matches(wl)), 4),
+        "expected_tokens_per_step": round(expected_tokens_per_step_pipelined(r.k, wl["match"]) if r.pipe else
+                                          expected_tokens_per_step(r.k, wl["match"], branch_matches(wl)), 4),
         "steps_per_generation": steps_per_gen,
         "step_hbm": {"bytes": int(step_bytes), "achieved_gbs": round(step_gbs, 1),
                      "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4),
@@ -562,6 +592,9 @@ def run_ours(args, wl, rank, world):
         "e2e": e2e, "gpu_launches": gpu_launches, "device_error_flags": flags,
         "prefill": prefill_line(r),
     }
+    if r.pipe:
+        out["config"].update({"pipelined": True, "note": "pipelined variant (not a step of the paper): every "
+                              "block is [y, k drafts, k adaptive tokens]; one forward per step"})
     if r.tree:
         out["config"].update({"tree_width": r.width, "q2": r.q2,
                               "tree": "width chains of k drafts below the root (Sec. 2.1.2)"})
@@ -610,6 +643,8 @@ def run_e2e(r, steps, steps_per_gen):
     tokens = 0
     h2d = d2h = 0
     st = torch.cuda.current_stream()
+    if r.pipe:
+        return run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start)
     t0 = time.perf_counter()
     for i in range(steps):
         j = i % steps_per_gen
@@ -643,6 +678,54 @@ def run_e2e(r, steps, steps_per_gen):
             lens[s] += a[s]
         tokens += sum(a)
         h2d += b * q * 4
+        d2h += b * q * 4 + b * 4
+    t1 = time.perf_counter()
+    return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d / steps, 1),
+            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": "eager C-ABI calls, host sync each step"}
+
+
+def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start):
+    """run_e2e for the pipelined variant: the host keeps each sequence's block mode, builds
+    [x_0, drafts or adaptive ids, adaptive ids] and copies the per-sequence verify counts in."""
+    import torch
+    b, k, q = r.b, r.k, r.q
+    nv_h = torch.zeros(b, dtype=torch.int32).pin_memory()
+    lens, last_out, last_acc = start()
+    prev_mode = [1] * b
+    tokens = h2d = d2h = 0
+    st = torch.cuda.current_stream()
+    t0 = time.perf_counter()
+    for i in range(steps):
+        if i % steps_per_gen == 0 and i > 0:
+            r.reset()
+            lens, last_out, last_acc = start()
+            prev_mode = [1] * b
+        blk, nv = [], []
+        for s in range(b):
+            a_mode = prev_mode[s] == 0 or last_acc[s] == k + 1
+            x0 = last_out[s][last_acc[s] - 1]
+            mid = [int(table[0, s, lens[s] + jj]) for jj in range(1, k + 1)] if a_mode else adaptive
+            blk += [x0] + mid + adaptive
+            nv.append(k if a_mode else 0)
+            prev_mode[s] = 1 if a_mode else 0
+        tok_h[:b * q].copy_(torch.tensor(blk, dtype=torch.int32))
+        nv_h.copy_(torch.tensor(nv, dtype=torch.int32))
+        r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
+        r.pnver.copy_(nv_h, non_blocking=True)
+        r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
+        wl = r.wl
+        r.ctx.accept_pipelined(r.kv, r.logits, r.toks, r.pnver, b, q, r.acc, r.out, temperature=wl["temperature"],
+                               top_p=wl["top_p"], seed=1234, top_k=wl["top_k"])
+        out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
+        acc_h.copy_(r.acc, non_blocking=True)
+        st.synchronize()
+        o, a = out_h.tolist(), acc_h.tolist()
+        for s in range(b):
+            last_out[s] = o[s * q:(s + 1) * q]
+            last_acc[s] = a[s]
+            lens[s] += a[s]
+        tokens += sum(a)
+        h2d += b * q * 4 + b * 4
         d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
     return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d / steps, 1),
@@ -697,12 +780,22 @@ def oracle_sample(shape_name, wl, weights_gpu=None, n_layers=2, repeat=1, gen_de
 
 
 def mean_rows(wl):
-    """Block rows of the workload's average step (steps alternate k + 1 and 1 + width * k rows)."""
+    """Block rows of the workload's average step (steps alternate k + 1 and 1 + width * k rows;
+    pipelined blocks have 2k + 1)."""
+    if wl.get("pipelined"):
+        return 2 * wl["k"] + 1
     return round((wl["k"] + 1 + 1 + wl.get("width", 1) * wl["k"]) / 2)
 
 
+def workload_tokens_per_step(wl):
+    """The stub's expected tokens per block step for the workload."""
+    if wl.get("pipelined"):
+        return expected_tokens_per_step_pipelined(wl["k"], wl["match"])
+    return expected_tokens_per_step(wl["k"], wl["match"], branch_matches(wl))
+
+
 def cpu_baseline(args, wl, weights_gpu):
-    tps = expected_tokens_per_step(wl["k"], wl["match"], branch_matches(wl))
+    tps = workload_tokens_per_step(wl)
     dev = next(iter(weights_gpu["layers"][0].values())).device if weights_gpu is not None else "cpu"
     t_step, det = oracle_sample(wl["shape"], wl, weights_gpu, n_layers=2, gen_device=dev)
     return {"value": round(tps / t_step, 4), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
@@ -720,7 +813,7 @@ def run_reference(args, wl, rank, world):
     import synth
     from oracle import model as OM
     shape = synth.SHAPES[wl["shape"]]
-    tps = expected_tokens_per_step(wl["k"], wl["match"], branch_matches(wl))
+    tps = workload_tokens_per_step(wl)
     q = mean_rows(wl)
     P = wl["prompt"]
     W = OM.Weights(shape, provider=lambda n, l: synth.make_weight(shape, n, l, 0, "cpu"), cache=True)

@@ -287,6 +287,45 @@ SDSAT_API sdsat_status sdsat_build_tree_block(sdsat_ctx* ctx, sdsat_kv* kv, int 
                                               const int32_t* draft_tables_dev, int width, int table_stride, int b,
                                               int k, int32_t* tokens_out_dev);
 
+/* ---- pipelined variant (not a step of the paper) ---------------------------------- */
+/* The verification block also carries the k adaptive tokens, so that a loop whose
+ * drafts are all accepted needs no separate draft step 1.  Every block has
+ * q = 2k + 1 rows [x_0, r_1 .. r_k, a_1 .. a_k] at slots len[s] .. len[s] + 2k:
+ *   mode A (drafts known): r_i = the drafts for positions len[s] + i; Eq. 3 verifies
+ *     them; if all k are accepted, the adaptive rows' targets are the next block's
+ *     drafts and the next block is mode A again, otherwise it is mode S;
+ *   mode S: r_i = a_i (the block is draft step 1 with k extra adaptive rows), nothing
+ *     is verified, t_0 is emitted and t_1 .. t_k are the next block's drafts (mode A).
+ * The emitted tokens are those of the two-step loop (and of plain decoding under greedy
+ * selection or the position-keyed sampler). */
+
+/* Build the next pipelined block on the device from the previous one's accept outputs:
+ *   prev_out_dev int32 [b*(2k+1)], prev_acc_dev int32 [b]: the previous accept call's
+ *     out_tokens and accepted_len (before the first block: out[s*(2k+1)] = the newest
+ *     prompt token, acc = 1, mode = 1);
+ *   mode_dev int32 [b], in: the previous block's mode (0 S, 1 A), out: this block's;
+ *   n_verify_dev int32 [b], out: k for mode A, 0 for mode S (for sdsat_accept_pipelined);
+ *   draft_table_dev: optional per-position drafts, [s*table_stride + len[s] + i] for
+ *     row i of a mode-A block (the harness's stub); otherwise the previous targets.
+ * x_0 = prev_out[s*(2k+1) + acc - 1]; mode A's drafts without a table are
+ * prev_out[s*(2k+1) + acc .. + acc + k - 1].  tokens_out_dev int32 [b*(2k+1)].
+ * Errors: EINVAL (null pointer, 2k + 1 > SDSAT_MAX_Q, b*(2k+1) > SDSAT_MAX_ROWS,
+ * table_stride < max_len + SDSAT_MAX_Q). */
+SDSAT_API sdsat_status sdsat_build_pipelined_block(sdsat_ctx* ctx, sdsat_kv* kv, const int32_t* prev_out_dev,
+                                                   const int32_t* prev_acc_dev, int32_t* mode_dev,
+                                                   int32_t* n_verify_dev, const int32_t* draft_table_dev,
+                                                   int table_stride, int b, int k, int32_t* tokens_out_dev);
+
+/* Target selection (argmax for temperature == 0, else the sampler of
+ * sdsat_accept_nucleus), Eq. 3 verification of n_verify_dev[s] drafts per sequence
+ * (device values, clamped to [0, q-1]) and the KV commit, as sdsat_accept_nucleus.
+ * Errors: EINVAL (null n_verify_dev, temperature < 0 or NaN, q < 2, the
+ * sdsat_accept_nucleus conditions), EUNSUPPORTED. */
+SDSAT_API sdsat_status sdsat_accept_pipelined(sdsat_ctx* ctx, sdsat_kv* kv, const float* logits_dev,
+                                              const int32_t* tokens_dev, const int32_t* n_verify_dev, int b, int q,
+                                              float temperature, float top_p, uint64_t rng_seed, int top_k,
+                                              int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit);
+
 /* Run n prompt tokens of sequence `seq` through the model and commit them
  * (len[seq] += n): the step before the decode loop.  Chunks of up to
  * SDSAT_MAX_ROWS positions go through one block forward each (the weights stream

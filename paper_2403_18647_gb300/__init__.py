@@ -91,6 +91,8 @@ def _lib():
             "sdsat_block_forward_tree": [P, P, P, P, I, I, P],
             "sdsat_accept_tree": [P, P, P, P, P, I, I, F, F, U64, I, P, P, P, I],
             "sdsat_build_tree_block": [P, P, I, P, I, P, P, I, I, I, I, P],
+            "sdsat_build_pipelined_block": [P, P, P, P, P, P, P, I, I, I, P],
+            "sdsat_accept_pipelined": [P, P, P, P, P, I, I, F, F, U64, I, P, P, I],
             "sdsat_prefill": [P, P, I, P, I],
             "sdsat_get_error": [P, ctypes.POINTER(ctypes.c_uint32)],
             "sdsat_op_gemm": [P, P, I, I, P, I, P],
@@ -326,6 +328,22 @@ class Context:
         _check(_lib().sdsat_build_tree_block(self.handle, kv.handle, mode, _ptr(prev_out), prev_q, _ptr(prev_acc),
                                              _ptr(draft_tables), width, table_stride, b, k, _ptr(tokens_out)),
                "sdsat_build_tree_block")
+
+    # ---- pipelined variant ----
+    def build_pipelined_block(self, kv: KV, prev_out, prev_acc, mode, n_verify, tokens_out, b: int, k: int,
+                              draft_table=None, table_stride: int = 0):
+        self._bind_stream()
+        _check(_lib().sdsat_build_pipelined_block(self.handle, kv.handle, _ptr(prev_out), _ptr(prev_acc), _ptr(mode),
+                                                  _ptr(n_verify), _ptr(draft_table), table_stride, b, k,
+                                                  _ptr(tokens_out)), "sdsat_build_pipelined_block")
+
+    def accept_pipelined(self, kv: KV, logits, tokens, n_verify, b: int, q: int, accepted_len, out_tokens,
+                         temperature: float = 0.0, top_p: float = 1.0, seed: int = 0, top_k: int = 0,
+                         commit: bool = True):
+        self._bind_stream()
+        _check(_lib().sdsat_accept_pipelined(self.handle, kv.handle, _ptr(logits), _ptr(tokens), _ptr(n_verify), b, q,
+                                             temperature, top_p, seed, top_k, _ptr(accepted_len), _ptr(out_tokens),
+                                             int(commit)), "sdsat_accept_pipelined")
 
     def prefill(self, kv: KV, seq: int, tokens):
         self._bind_stream()

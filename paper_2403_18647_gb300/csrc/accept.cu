@@ -701,7 +701,8 @@ __global__ void __launch_bounds__(ACC_THREADS) accept_kernel(const AcceptParams 
   for (int i = 0; i < p.q; ++i) tg[i] = __ldcg(p.targets + sl * p.q + i);
   int m = 0;
   if (!p.parent) {
-    for (int i = 1; i <= p.n_verify; ++i) {        // Eq. 3: prefix of matching drafts
+    const int nv = p.n_verify_dev ? min(max(__ldcg(p.n_verify_dev + sl), 0), p.q - 1) : p.n_verify;
+    for (int i = 1; i <= nv; ++i) {                 // Eq. 3: prefix of matching drafts
       if (__ldcg(p.drafts + sl * p.q + i) != tg[i - 1]) break;
       m = i;
     }
@@ -856,8 +857,31 @@ __global__ void build_block_kernel(BuildParams b) {
   pdl_wait();
   pdl_trigger();
   const int sl = blockIdx.x, j = threadIdx.x;
-  if (j >= b.q) return;
   const int* prev = b.prev_out + sl * b.prev_q;
+  if (b.mode == 3) {
+    // pipelined blocks [x_0, r_1 .. r_k, a_1 .. a_k]: mode A (drafts known) after a mode-S
+    // block or after a mode-A block that accepted all k drafts, else mode S (r_i = a_i);
+    // x_0 = the newest emitted token, the drafts the k targets after it
+    const int acc = __ldcg(b.prev_acc + sl);
+    const bool a_mode = __ldcg(b.pipe_mode + sl) == 0 || acc == b.k + 1;
+    __syncthreads();   // every thread has read the previous mode before thread 0 replaces it
+    if (j == 0) {
+      b.pipe_mode[sl] = a_mode ? 1 : 0;
+      b.pipe_nverify[sl] = a_mode ? b.k : 0;
+    }
+    if (j >= b.q) return;
+    int t;
+    if (j == 0) {
+      t = __ldcg(prev + acc - 1);
+    } else if (j <= b.k && a_mode) {
+      t = b.table ? __ldcg(b.table + (size_t)sl * b.table_stride + __ldcg(b.len + sl) + j) : __ldcg(prev + acc - 1 + j);
+    } else {
+      t = b.adaptive[(j - 1) % b.k];
+    }
+    b.tokens[sl * b.q + j] = t;
+    return;
+  }
+  if (j >= b.q) return;
   int t;
   if (b.mode == 1) {
     t = (j == 0) ? __ldcg(prev + __ldcg(b.prev_acc + sl) - 1) : b.adaptive[j - 1];

@@ -193,6 +193,7 @@ struct AcceptParams {
   int* targets;             // scratch [nb*q]
   int* counters;            // scratch [nb], zero between launches
   long long* emitted;       // [B] tokens emitted per sequence (commit only), or null
+  const int* n_verify_dev;  // [nb] drafts verified per sequence (pipelined blocks); null: n_verify
   const int* parent;        // tree blocks: [nb*q] parent row of every row (row 0: -1); null = chain
   int* path;                // tree blocks: [nb*q] accepted path rows, -1 past its end (optional)
   int* tree_ws;             // tree blocks: [nb][TREE_WS_STRIDE] len before the step, m, path rows
@@ -211,8 +212,10 @@ struct BuildParams {
   int table_stride, table_batch;
   const int* len;           // [B] committed lengths
   const int* adaptive;      // [SDSAT_MAX_ADAPTIVE] adaptive token ids
-  int nb, q, k;             // q rows per sequence; mode 2: q = 1 + width * k
+  int nb, q, k;             // q rows per sequence; mode 2: q = 1 + width * k; mode 3: q = 2k + 1
   int* tokens;              // [nb][q]
+  int* pipe_mode;           // mode 3: [nb] in: the previous block's mode, out: this block's (0 S, 1 A)
+  int* pipe_nverify;        // mode 3: [nb] out: drafts this block verifies (k in mode A, 0 in S)
 };
 cudaError_t launch_build_block(const BuildParams& b, cudaStream_t st, bool pdl);
 // tree block rows: positions len + depth and the attention masks (ancestors and self)

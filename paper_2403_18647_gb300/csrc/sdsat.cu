@@ -520,7 +520,8 @@ sdsat_status prefill_chunk(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
 
 sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, const int32_t* drafts, int b, int q,
                            int n_verify, float top_p, float temperature, uint64_t seed, int top_k, int32_t* acc,
-                           int32_t* out, int commit, const int32_t* parent = nullptr, int32_t* path = nullptr) {
+                           int32_t* out, int commit, const int32_t* parent = nullptr, int32_t* path = nullptr,
+                           const int32_t* n_verify_dev = nullptr) {
   if (!c || !kv || kv->ctx != c || !logits || !drafts || !acc || !out) return SDSAT_EINVAL;
   if (b < 1 || b > kv->batch || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
   if (n_verify < 0 || n_verify >= q || top_k < 0) return SDSAT_EINVAL;
@@ -552,6 +553,7 @@ sdsat_status accept_common(sdsat_ctx* c, sdsat_kv* kv, const float* logits, cons
   p.emitted = kv->emitted;
   p.parent = parent;
   p.path = path;
+  p.n_verify_dev = n_verify_dev;
   p.tree_ws = c->tree_ws;
   if (timed(c, K_ACCEPT, [&] { return launch_accept(p, c->stream, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
   if (!parent) return SDSAT_OK;
@@ -877,6 +879,15 @@ sdsat_status sdsat_accept_tree(sdsat_ctx* c, sdsat_kv* kv, const float* logits_d
                        temperature, rng_seed, top_k, accepted_len_dev, out_tokens_dev, commit, parent_dev, path_dev);
 }
 
+sdsat_status sdsat_accept_pipelined(sdsat_ctx* c, sdsat_kv* kv, const float* logits_dev, const int32_t* tokens_dev,
+                                    const int32_t* n_verify_dev, int b, int q, float temperature, float top_p,
+                                    uint64_t rng_seed, int top_k, int32_t* accepted_len_dev, int32_t* out_tokens_dev,
+                                    int commit) {
+  if (!n_verify_dev || !(temperature >= 0.f) || q < 2) return SDSAT_EINVAL;
+  return accept_common(c, kv, logits_dev, tokens_dev, b, q, q - 1, temperature > 0.f ? top_p : 1.f, temperature,
+                       rng_seed, top_k, accepted_len_dev, out_tokens_dev, commit, nullptr, nullptr, n_verify_dev);
+}
+
 sdsat_status sdsat_kv_commit(sdsat_ctx* c, sdsat_kv* kv, const int32_t* new_len_dev, int b) {
   if (!c || !kv || kv->ctx != c || !new_len_dev || b < 1 || b > kv->batch || b > 64) return SDSAT_EINVAL;
   return timed(c, K_KV_COMMIT, [&] { return launch_commit(kv->len, new_len_dev, b, kv->cap, c->err, c->stream, c->pdl); }) ==
@@ -1011,6 +1022,23 @@ sdsat_status sdsat_build_tree_block(sdsat_ctx* c, sdsat_kv* kv, int mode, const 
   if (draft_tables_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
   BuildParams bp{mode, prev_out_dev, prev_q, prev_acc_dev, draft_tables_dev, table_stride, kv->batch, kv->len,
                  c->adaptive, b, q, k, tokens_out_dev};
+  return timed(c, K_BUILD_BLOCK, [&] { return launch_build_block(bp, c->stream, c->pdl); }) == cudaSuccess
+             ? SDSAT_OK
+             : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_build_pipelined_block(sdsat_ctx* c, sdsat_kv* kv, const int32_t* prev_out_dev,
+                                         const int32_t* prev_acc_dev, int32_t* mode_dev, int32_t* n_verify_dev,
+                                         const int32_t* draft_table_dev, int table_stride, int b, int k,
+                                         int32_t* tokens_out_dev) {
+  if (!c || !kv || kv->ctx != c || !prev_out_dev || !prev_acc_dev || !mode_dev || !n_verify_dev || !tokens_out_dev)
+    return SDSAT_EINVAL;
+  const int q = 2 * k + 1;
+  if (b < 1 || b > kv->batch || k < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS) return SDSAT_EINVAL;
+  if (c->cfg.n_adaptive > 1 && k > c->cfg.n_adaptive) return SDSAT_EINVAL;
+  if (draft_table_dev && table_stride < kv->cap + SDSAT_MAX_Q) return SDSAT_EINVAL;
+  BuildParams bp{3, prev_out_dev, q, prev_acc_dev, draft_table_dev, table_stride, kv->batch, kv->len,
+                 c->adaptive, b, q, k, tokens_out_dev, mode_dev, n_verify_dev};
   return timed(c, K_BUILD_BLOCK, [&] { return launch_build_block(bp, c->stream, c->pdl); }) == cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;

@@ -16,7 +16,8 @@ def test_header_declares_the_boundary():
     names = _declared()
     for n in ("sdsat_create", "sdsat_destroy", "sdsat_kv_create", "sdsat_block_forward",
               "sdsat_accept_greedy", "sdsat_accept_nucleus", "sdsat_kv_commit", "sdsat_status_string",
-              "sdsat_block_forward_tree", "sdsat_accept_tree", "sdsat_build_tree_block"):
+              "sdsat_block_forward_tree", "sdsat_accept_tree", "sdsat_build_tree_block",
+              "sdsat_build_pipelined_block", "sdsat_accept_pipelined"):
         assert n in names
 
 
@@ -46,3 +47,5 @@ def test_argument_errors_are_synchronous_and_need_no_gpu():
     assert lib.sdsat_block_forward_tree(None, None, None, None, 1, 7, None) == 1
     assert lib.sdsat_accept_tree(None, None, None, None, None, 1, 7, 0.0, 1.0, 0, 0, None, None, None, 1) == 1
     assert lib.sdsat_build_tree_block(None, None, 2, None, 4, None, None, 2, 0, 1, 3, None) == 1
+    assert lib.sdsat_build_pipelined_block(None, None, None, None, None, None, None, 0, 1, 5, None) == 1
+    assert lib.sdsat_accept_pipelined(None, None, None, None, None, 1, 11, 0.0, 1.0, 0, 0, None, None, 1) == 1
