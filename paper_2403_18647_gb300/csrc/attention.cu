@@ -4,9 +4,9 @@
 // [0, len[s]) and to block rows 0..j (slots len[s] .. len[s]+j), which the QKV
 // epilogue has just written; this is how Eq. 1-2 evaluate every appended
 // position of the block in one pass.  A tree block (Sec. 2.1.2) replaces the
-// rows 0..j by row j's ancestors and itself, given as one bit mask per row.  A
-// prefill chunk of one sequence runs as consecutive groups of q rows: group g
-// sees len + g*q committed slots, then its rows causally.
+// rows 0..j by row j's ancestors and itself, given as one bit mask per row.
+// (Prefill attention, many query rows per sequence, is a separate kernel at the
+// end of this file.)
 // The bytes are the K and V rows (bf16, hd*2 bytes each), read once per
 // (sequence, head) for all q rows together.
 //
@@ -126,7 +126,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   // first kernel (RMSNorm) lets its dependents launch only after every earlier kernel
   // has completed.  Slots below them are not written during this forward either.
   if (tid < p.nb) {
-    const int len = p.groups ? __ldcg(p.len + p.seq0) + tid * q : __ldcg(p.len + p.seq0 + tid);
+    const int len = __ldcg(p.len + p.seq0 + tid);
     len_seq[tid] = len;
     nu_seq[tid] = (min(len + q, p.cap) + ATT_UNIT - 1) / ATT_UNIT;
   }
@@ -164,10 +164,8 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   auto unit_row = [&](int u, bool& committed) {
     int s, hh, cc;
     locate(u, s, hh, cc);
-    // (prefill groups: the slots after the sequence's committed length are this chunk's rows,
-    // written by the kernel before)
-    committed = (cc + 1) * ATT_UNIT <= (p.groups ? len_seq[0] : len_seq[s]);
-    return p.row0 + ((p.seq0 + (p.groups ? 0 : s)) * H + hh) * p.cap + cc * ATT_UNIT;
+    committed = (cc + 1) * ATT_UNIT <= len_seq[s];
+    return p.row0 + ((p.seq0 + s) * H + hh) * p.cap + cc * ATT_UNIT;
   };
   uint64_t pol = 0;
   auto issue = [&](int k, int row) {   // unit u0 + k into stage k % ATT_STAGES
@@ -555,6 +553,226 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     trace_write(p.trace, merges | ((unsigned)n << 8), t_entry, t_wait, t_k, t_part, t_merge, globaltimer_ns());
 }
 
+// ---- prefill attention ----------------------------------------------------------------
+// Causal attention of a prefill chunk over the cache (flash attention, mma.sync m16n8k16).
+// One CTA per (head, block of 64 chunk positions), heaviest blocks first; four warps of 16
+// query rows each.  Units of 64 keys stream through a two-stage TMA ring (the decode
+// kernel's tiles).  Per unit and warp: S = Q K^T (16 rows x 64 keys; Q as bf16 hi + lo, both
+// products into one accumulator), the causal mask on the units that reach the block's
+// positions, the online-softmax update (row max over the four lanes of a row), then
+// O = O * alpha + P V with P taken straight from the S accumulators as the A operand (bf16
+// hi + lo) and V through transposed ldmatrix loads.
+template <int HD>
+struct PfAttCfg {
+  static constexpr int QS = HD * 2 + 16;                             // bytes per Q row (padded)
+  static constexpr size_t OFF_Q = (size_t)ATT_STAGES * AttCfg<HD>::STAGE;
+  static constexpr size_t OFF_BAR = OFF_Q + 2 * 64 * QS;
+  static constexpr size_t SMEM = 1024 + OFF_BAR + ATT_STAGES * 8 + 16;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(128) prefill_attention_kernel(const __grid_constant__ PfAttnParams p) {
+  using C = AttCfg<HD>;
+  using F = PfAttCfg<HD>;
+  constexpr int KSTEPS = HD / 16;   // k-steps of Q K^T over the head dimension
+  constexpr int NT = HD / 8;        // 8-dimension tiles of O
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* Qh = smem + F::OFF_Q;          // bf16 [64][HD] scaled q, hi part (padded rows)
+  uint8_t* Ql = Qh + 64 * F::QS;          // lo part
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + F::OFF_BAR);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(full + ATT_STAGES);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, tig = lane & 3;
+  const int mi = lane >> 3, r8 = lane & 7;
+  const int NQB = (p.M + 63) / 64;
+  const int qb = NQB - 1 - (int)blockIdx.x / p.H, h = (int)blockIdx.x % p.H;
+  const int q0 = qb * 64;
+  if (tid == 0) {
+    for (int s = 0; s < ATT_STAGES; ++s) mbar_init(&full[s], 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  pdl_wait();   // q and this chunk's K / V rows come from the kernels before
+  pdl_trigger();
+  const int len = __ldcg(p.len + p.seq);
+  const int kend = len + min(q0 + 64, p.M);    // keys this block's positions may see
+  const int nu = (kend + ATT_UNIT - 1) / ATT_UNIT;
+  const int rowbase = p.row0 + (p.seq * p.H + h) * p.cap;
+  __syncthreads();
+  auto issue = [&](int u) {
+    uint8_t* st = smem + (size_t)(u % ATT_STAGES) * C::STAGE;
+    uint64_t* bar = &full[u % ATT_STAGES];
+    mbar_arrive_expect_tx(bar, C::STAGE);
+#pragma unroll
+    for (int hh = 0; hh < C::HALVES; ++hh)
+      tma_load_2d(st + hh * C::HALF_BYTES, &p.kmap, bar, hh * 64, rowbase + u * ATT_UNIT, l2_policy_evict_last());
+#pragma unroll
+    for (int hh = 0; hh < C::HALVES; ++hh)
+      tma_load_2d(st + C::TILE + hh * C::HALF_BYTES, &p.vmap, bar, hh * 64, rowbase + u * ATT_UNIT,
+                  l2_policy_evict_last());
+  };
+  if (tid == 0) {
+    tma_prefetch_desc(&p.kmap);
+    tma_prefetch_desc(&p.vmap);
+    for (int u = 0; u < min(nu, ATT_STAGES); ++u) issue(u);
+  }
+  // the block's queries, scaled by 1/sqrt(hd), as bf16 hi + lo (positions >= M: zero)
+  const float scale = rsqrtf((float)HD);
+  for (int i = tid; i < 64 * (HD / 2); i += 128) {
+    const int j = i / (HD / 2), d = (i % (HD / 2)) * 2;
+    float x0 = 0.f, x1 = 0.f;
+    if (q0 + j < p.M) {
+      const float2 v = __ldcg(reinterpret_cast<const float2*>(p.Q + (size_t)(q0 + j) * p.q_ld + h * HD + d));
+      x0 = v.x * scale;
+      x1 = v.y * scale;
+    }
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
+    *reinterpret_cast<uint32_t*>(Qh + j * F::QS + d * 2) =
+        (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+    *reinterpret_cast<uint32_t*>(Ql + j * F::QS + d * 2) = pack_bf16(x0 - __bfloat162float(h0), x1 - __bfloat162float(h1));
+  }
+  __syncthreads();
+
+  const int wr = warp * 16;                            // this warp's first row in the block
+  const int pos0 = len + q0 + wr + g;                  // absolute position of row g (row g + 8: +8)
+  float O[NT][4];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) O[nt][0] = O[nt][1] = O[nt][2] = O[nt][3] = 0.f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  for (int u = 0; u < nu; ++u) {
+    const uint8_t* Kt = smem + (size_t)(u % ATT_STAGES) * C::STAGE;
+    const uint8_t* Vt = Kt + C::TILE;
+    const bool ok = mbar_wait_bounded(&full[u % ATT_STAGES], (u / ATT_STAGES) & 1, abort_flag, p.err);
+    __syncwarp();
+    float s[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+    if (ok) {
+#pragma unroll
+      for (int ks = 0; ks < KSTEPS; ++ks) {
+        uint32_t ah0, ah1, ah2, ah3, al0, al1, al2, al3;
+        const int qrow = wr + r8 + 8 * (mi & 1), qcol = ks * 16 + 8 * (mi >> 1);
+        ldsm_x4(smem_u32(Qh + qrow * F::QS + qcol * 2), ah0, ah1, ah2, ah3);
+        ldsm_x4(smem_u32(Ql + qrow * F::QS + qcol * 2), al0, al1, al2, al3);
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          const int key = np * 16 + r8 + 8 * (mi >> 1);
+          const int c = ks * 2 + (mi & 1), hh = c >> 3, cc = c & 7;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(smem_u32(Kt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), b0, b1, b2, b3);
+          mma_bf16_16816(s[2 * np], ah0, ah1, ah2, ah3, b0, b1);
+          mma_bf16_16816(s[2 * np], al0, al1, al2, al3, b0, b1);
+          mma_bf16_16816(s[2 * np + 1], ah0, ah1, ah2, ah3, b2, b3);
+          mma_bf16_16816(s[2 * np + 1], al0, al1, al2, al3, b2, b3);
+        }
+      }
+    }
+    // causal mask: key slot kp is visible to the row at position pos iff kp <= pos
+    const int kbase = u * ATT_UNIT;
+    const bool need_mask = !ok || kbase + ATT_UNIT - 1 > pos0 - g;   // some key passes the warp's first row
+    if (need_mask) {
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int kp = kbase + nt * 8 + 2 * tig + (e & 1);
+          if (!ok || kp > pos0 + 8 * (e >> 1)) s[nt][e] = -INFINITY;
+        }
+    }
+    // online softmax: rows g (e = 0, 1) and g + 8 (e = 2, 3); the four lanes of a row share it
+    float alpha[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(s[nt][2 * r], s[nt][2 * r + 1]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float mn = fmaxf(mrow[r], mx);
+      alpha[r] = (mn == -INFINITY) ? 1.f : __expf(mrow[r] - mn);
+      mrow[r] = mn;
+    }
+    float rs[2] = {0.f, 0.f};
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float v = (s[nt][e] == -INFINITY) ? 0.f : __expf(s[nt][e] - mrow[e >> 1]);
+        s[nt][e] = v;
+        rs[e >> 1] += v;
+      }
+    lrow[0] = lrow[0] * alpha[0] + rs[0];
+    lrow[1] = lrow[1] * alpha[1] + rs[1];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      O[nt][0] *= alpha[0];
+      O[nt][1] *= alpha[0];
+      O[nt][2] *= alpha[1];
+      O[nt][3] *= alpha[1];
+    }
+    // O += P V, k-steps of 16 keys; P's A fragments are the S accumulators of two key tiles
+    if (ok) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint32_t ph[4], pl[4];
+        const float* s0 = s[2 * j];
+        const float* s1 = s[2 * j + 1];
+        const float pv[8] = {s0[0], s0[1], s0[2], s0[3], s1[0], s1[1], s1[2], s1[3]};
+#pragma unroll
+        for (int f = 0; f < 4; ++f) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(pv[2 * f]), h1 = __float2bfloat16_rn(pv[2 * f + 1]);
+          ph[f] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+          pl[f] = pack_bf16(pv[2 * f] - __bfloat162float(h0), pv[2 * f + 1] - __bfloat162float(h1));
+        }
+        // A fragment order: (row g, keys 0-7), (row g+8, keys 0-7), (row g, keys 8-15), (row g+8, keys 8-15)
+#pragma unroll
+        for (int dp = 0; dp < NT / 2; ++dp) {
+          const int key = j * 16 + r8 + 8 * (mi & 1);
+          const int dim = dp * 16 + 8 * (mi >> 1);
+          const int hh = dim >> 6, cc = (dim & 63) >> 3;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), b0, b1, b2, b3);
+          mma_bf16_16816(O[2 * dp], ph[0], ph[1], ph[2], ph[3], b0, b1);
+          mma_bf16_16816(O[2 * dp], pl[0], pl[1], pl[2], pl[3], b0, b1);
+          mma_bf16_16816(O[2 * dp + 1], ph[0], ph[1], ph[2], ph[3], b2, b3);
+          mma_bf16_16816(O[2 * dp + 1], pl[0], pl[1], pl[2], pl[3], b2, b3);
+        }
+      }
+    }
+    __syncthreads();   // every warp is done with the stage
+    if (tid == 0 && u + ATT_STAGES < nu && !*abort_flag) issue(u + ATT_STAGES);
+  }
+  if (*abort_flag && tid == 0) {   // let the copies in flight land before the CTA exits
+    for (int u = max(0, nu - ATT_STAGES); u < nu; ++u) {
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(&full[u % ATT_STAGES], (u / ATT_STAGES) & 1))
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) break;
+    }
+  }
+  // O / L for the rows of this block inside the chunk, fp32 and bf16 hi + lo
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    float l = lrow[r];
+    l += __shfl_xor_sync(0xffffffffu, l, 1);
+    l += __shfl_xor_sync(0xffffffffu, l, 2);
+    const float inv = l > 0.f ? 1.0f / l : 0.f;
+    const int row = q0 + wr + g + 8 * r;
+    if (row >= p.M) continue;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const float o0 = O[nt][2 * r] * inv, o1 = O[nt][2 * r + 1] * inv;
+      const size_t idx = (size_t)row * p.out_ld + h * HD + nt * 8 + 2 * tig;
+      *reinterpret_cast<float2*>(p.out + idx) = make_float2(o0, o1);
+      const __nv_bfloat16 h0 = __float2bfloat16_rn(o0), h1 = __float2bfloat16_rn(o1);
+      *reinterpret_cast<uint32_t*>(p.out_hi + idx) =
+          (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+      *reinterpret_cast<uint32_t*>(p.out_lo + idx) = pack_bf16(o0 - __bfloat162float(h0), o1 - __bfloat162float(h1));
+    }
+  }
+}
+
 size_t attention_smem_bytes(int hd) { return hd == 64 ? AttCfg<64>::SMEM : AttCfg<128>::SMEM; }
 
 cudaError_t attention_prepare() {
@@ -563,7 +781,9 @@ cudaError_t attention_prepare() {
   if ((e = cudaFuncSetAttribute(attention_kernel<64, 1>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
   if ((e = cudaFuncSetAttribute(attention_kernel<64, 2>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
   if ((e = cudaFuncSetAttribute(attention_kernel<128, 1>, a, (int)AttCfg<128>::SMEM)) != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attention_kernel<128, 2>, a, (int)AttCfg<128>::SMEM);
+  if ((e = cudaFuncSetAttribute(attention_kernel<128, 2>, a, (int)AttCfg<128>::SMEM)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(prefill_attention_kernel<64>, a, (int)PfAttCfg<64>::SMEM)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(prefill_attention_kernel<128>, a, (int)PfAttCfg<128>::SMEM);
 }
 
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl) {
@@ -584,6 +804,21 @@ cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, 
   const bool one = p.q <= 8;
   if (p.hd == 64) return one ? cudaLaunchKernelEx(&cfg, attention_kernel<64, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<64, 2>, p);
   return one ? cudaLaunchKernelEx(&cfg, attention_kernel<128, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<128, 2>, p);
+}
+
+cudaError_t launch_prefill_attention(const PfAttnParams& p, cudaStream_t st, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(((p.M + 63) / 64) * p.H);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = p.hd == 64 ? PfAttCfg<64>::SMEM : PfAttCfg<128>::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return p.hd == 64 ? cudaLaunchKernelEx(&cfg, prefill_attention_kernel<64>, p)
+                    : cudaLaunchKernelEx(&cfg, prefill_attention_kernel<128>, p);
 }
 
 }  // namespace sdsat

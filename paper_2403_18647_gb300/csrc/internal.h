@@ -119,8 +119,6 @@ struct AttnParams {
   const int* len;       // [B]
   const uint32_t* anc;  // [nb*q] tree blocks: bit i of row j = row j attends block row i; null = causal
   int seq0, nb, q, H, hd, cap;
-  int groups;           // prefill: the nb "sequences" are consecutive groups of q rows of sequence
-                        //   seq0 (group g sees len[seq0] + g*q committed slots, then causal)
   float* out;           // [rows][out_ld] fp32
   int out_ld;
   __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
@@ -135,6 +133,24 @@ size_t attention_smem_bytes(int hd);
 cudaError_t attention_prepare();   // set smem attributes (idempotent)
 // grid: min(2 * num_sms, 14 * H) CTAs, so at most ATT_SEG_MAX CTAs share one (sequence, head)
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl);
+
+// Causal attention of M consecutive prompt positions of sequence seq (a prefill chunk at
+// slots len[seq] .. len[seq]+M-1, already in the cache) over the cache: position i sees
+// slots [0, len + i].  One CTA per (head, 64-position block).
+struct PfAttnParams {
+  CUtensorMap kmap, vmap;   // the caches, as AttnParams
+  int row0;                 // first cache row of this layer
+  const float* Q;           // [M][q_ld] rotated queries, head h at column h*hd
+  int q_ld;
+  const int* len;
+  int seq, M, H, hd, cap;
+  float* out;               // [M][out_ld] fp32
+  int out_ld;
+  __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
+  __nv_bfloat16* out_lo;
+  uint32_t* err;
+};
+cudaError_t launch_prefill_attention(const PfAttnParams& p, cudaStream_t st, bool pdl);
 
 // ---- prefill (prompt chunks of up to PF_ROWS positions) -------------------------
 constexpr int PF_ROWS = 512;

@@ -88,12 +88,12 @@ struct LayerMaps {
 enum KClass : int {
   K_RMSNORM = 0, K_GEMM_QKV, K_ATTENTION, K_GEMM_O, K_GEMM_GATEUP, K_GEMM_DOWN, K_GEMM_LM_HEAD, K_ACCEPT,
   K_BUILD_BLOCK, K_KV_COMMIT, K_PREFILL_COMMIT, K_GEMM_OP, K_ATTENTION_OP, K_TREE_PREP, K_TREE_COMPACT,
-  K_PF_GEMM, K_PF_ROPE_KV, K_COUNT
+  K_PF_GEMM, K_PF_ROPE_KV, K_PF_ATTENTION, K_COUNT
 };
 const char* const KCLASS_NAME[K_COUNT] = {"rmsnorm", "gemm_qkv", "attention", "gemm_o", "gemm_gateup", "gemm_down",
                                           "gemm_lm_head", "accept", "build_block", "kv_commit", "prefill_commit",
                                           "gemm_op", "attention_op", "tree_prep", "tree_compact", "prefill_gemm",
-                                          "prefill_rope_kv"};
+                                          "prefill_rope_kv", "prefill_attention"};
 
 constexpr int MAX_GEMM_TILES = 1 << 16;
 constexpr int OP_MAX_K = 32768;   // K limit of sdsat_op_gemm (its operand scratch is sized at create)
@@ -138,9 +138,6 @@ struct sdsat_ctx {
   float* pf_qkv = nullptr;       // [PF_ROWS][3R] projections before RoPE
   float* pf_q = nullptr;         // [PF_ROWS][R] rotated queries
   float* pf_attn = nullptr;      // [PF_ROWS][R] attention output
-  float* pf_part_o = nullptr;    // attention partials for PF_ROWS rows
-  float* pf_part_ml = nullptr;
-  int* pf_att_counters = nullptr;
   __nv_bfloat16* pf_hi[X_COUNT] = {};   // GEMM operands [PF_ROWS][K] (normed x, attention, act)
   __nv_bfloat16* pf_lo[X_COUNT] = {};
   CUtensorMap pf_xmap[X_COUNT][2];      // boxes of 64 x 128
@@ -453,8 +450,8 @@ sdsat_status prefill_chunk(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
     RopeKvParams rp{c->pf_qkv, c->pf_q, kv->k + l * layer_elems, kv->v + l * layer_elems, kv->len, seq, H, hd,
                     kv->cap, c->rope, cf.max_position, c->err};
     if (timed(c, K_PF_ROPE_KV, [&] { return launch_rope_kv(rp, M, st, c->pdl); }) != cudaSuccess) return SDSAT_ECUDA;
-    // attention: the chunk as causal groups of SDSAT_MAX_Q positions over the cache
-    AttnParams a;
+    // causal attention of the chunk's positions over the cache
+    PfAttnParams a;
     std::memset(&a, 0, sizeof(a));
     a.kmap = kv->kmap;
     a.vmap = kv->vmap;
@@ -462,10 +459,8 @@ sdsat_status prefill_chunk(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
     a.Q = c->pf_q;
     a.q_ld = R;
     a.len = kv->len;
-    a.groups = 1;
-    a.seq0 = seq;
-    a.nb = M / SDSAT_MAX_Q;
-    a.q = SDSAT_MAX_Q;
+    a.seq = seq;
+    a.M = M;
     a.H = H;
     a.hd = hd;
     a.cap = kv->cap;
@@ -473,12 +468,8 @@ sdsat_status prefill_chunk(sdsat_ctx* c, sdsat_kv* kv, int seq, const int32_t* t
     a.out_ld = R;
     a.out_hi = c->pf_hi[X_ATTN];
     a.out_lo = c->pf_lo[X_ATTN];
-    a.part_o = c->pf_part_o;
-    a.part_ml = c->pf_part_ml;
-    a.counters = c->pf_att_counters;
     a.err = c->err;
-    a.trace = next_trace(c, K_ATTENTION);
-    if (timed(c, K_ATTENTION, [&] { return launch_attention(a, c->num_sms, st, c->pdl); }) != cudaSuccess)
+    if (timed(c, K_PF_ATTENTION, [&] { return launch_prefill_attention(a, st, c->pdl); }) != cudaSuccess)
       return SDSAT_ECUDA;
     PfGemmParams go = base(X_ATTN, R);
     go.tmap[0] = mp.o;
@@ -674,11 +665,9 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
            make_xmap(&c->xmap[xs][mi][1], c->x_lo[xs], rows, xcols[xs], 16 << mi);
   }
   if (ok && c->has_weights) {
-    const int pr = PF_ROWS, H = cfg->n_heads, hd = cfg->head_dim;
+    const int pr = PF_ROWS;
     ok = dalloc(c, &c->pf_h, (size_t)pr * d) && dalloc(c, &c->pf_qkv, (size_t)pr * 3 * R) &&
-         dalloc(c, &c->pf_q, (size_t)pr * R) && dalloc(c, &c->pf_attn, (size_t)pr * R) &&
-         dalloc(c, &c->pf_part_o, (size_t)pr * H * ATT_SEG_MAX * hd) &&
-         dalloc(c, &c->pf_part_ml, (size_t)pr * H * ATT_SEG_MAX * 2) && dalloc(c, &c->pf_att_counters, (size_t)pr * H);
+         dalloc(c, &c->pf_q, (size_t)pr * R) && dalloc(c, &c->pf_attn, (size_t)pr * R);
     for (int xs = 0; ok && xs < X_COUNT; ++xs)
       ok = dalloc(c, &c->pf_hi[xs], (size_t)pr * xcols[xs]) && dalloc(c, &c->pf_lo[xs], (size_t)pr * xcols[xs]) &&
            make_xmap(&c->pf_xmap[xs][0], c->pf_hi[xs], pr, xcols[xs], 128) &&
