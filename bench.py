@@ -617,7 +617,8 @@ def prefill_line(r, chunk=512):
     tf = flops / sec / 1e12
     return {"tokens": n, "ms": round(r.prefill_ms, 3), "tokens_per_s": round(n / sec, 1), "chunk_rows": chunk,
             "tflops": round(tf, 1), "frac_of_measured_bf16": round(tf / tpk, 4), "peak": tpk, "peak_source": kind,
-            "note": "tiled tcgen05 GEMM (128 weight rows x 128 positions), attention in 16-row causal groups"}
+            "note": "tiled tcgen05 GEMM (128 weight rows x 128 positions), causal flash attention over "
+                    "64-position blocks"}
 
 
 def run_e2e(r, steps, steps_per_gen):

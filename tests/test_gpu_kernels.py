@@ -304,3 +304,39 @@ def test_accept_nucleus_list_and_block_paths(accept_env, T, top_p, top_k):
     _, rout = _oracle_accept(lgc, drafts, 1, n, 0, [40], T, top_p, 3, top_k)
     assert out == rout
     assert flags == 0
+
+
+@pytest.mark.parametrize("N,K", [(15360, 5120), (27648, 5120), (5120, 13824), (32016, 5120)])
+def test_gemm_13b_shapes_sampled(tiny_ctx, N, K):
+    """The 13B model's projection shapes (QKV, gate+up, down, LM head) at M = 6; 384 sampled
+    output columns against fp64 dot products."""
+    M = 6
+    x = synth.normal_f32(4, M, (M, K), 1.0, device="cuda")
+    w = synth.normal_bf16(4, N + K, (N, K), 0.02, device="cuda")
+    y = torch.empty((M, N), device="cuda")
+    tiny_ctx.op_gemm(x, w, y)
+    torch.cuda.synchronize()
+    cols = torch.cat([torch.arange(0, 128), torch.randint(0, N, (128,), generator=torch.Generator().manual_seed(N)),
+                      torch.arange(N - 128, N)])
+    ref = OM.linear(x.cpu().double().numpy(), w[cols.cuda()].cpu().double().numpy())
+    err = np.abs(y[:, cols.cuda()].cpu().double().numpy() - ref).max()
+    assert err <= 5e-5 * math.sqrt(K) * 0.02 + 1e-6 * np.abs(ref).max(), err
+
+
+def test_attention_40_heads_sampled(big_ctx):
+    """40 heads (the 13B shape) at context 4096, q = 6: three sampled heads against the oracle."""
+    b, q, H, hd, n = 1, 6, 40, 128, 4096
+    cap = n + q
+    K = synth.normal_bf16(6, 1, (H * cap, hd), 1.0, device="cuda").reshape(1, H, cap, hd)
+    V = synth.normal_bf16(6, 2, (H * cap, hd), 1.0, device="cuda").reshape(1, H, cap, hd)
+    qm = synth.normal_f32(6, 3, (q, H * hd), 1.0, device="cuda")
+    ln = torch.tensor([n], dtype=torch.int32, device="cuda")
+    out = torch.empty((q, H * hd), device="cuda")
+    big_ctx.op_attention(qm, K, V, ln, b, q, H, hd, cap, out)
+    torch.cuda.synchronize()
+    for h in (0, 21, 39):
+        qs = qm.cpu().double().numpy().reshape(q, H, hd)[:, h:h + 1]
+        o = OM.attend(qs, K[0, h:h + 1].cpu().double().numpy(), V[0, h:h + 1].cpu().double().numpy(),
+                      [n + j + 1 for j in range(q)])
+        err = np.abs(out.cpu().double().numpy().reshape(q, H, hd)[:, h] - o[:, 0]).max()
+        assert err <= 2e-5, (h, err)
