@@ -621,11 +621,61 @@ def prefill_line(r, chunk=512):
                     "64-position blocks"}
 
 
+def step_calls(r):
+    """The C-ABI calls of one step once its block input is in place, by step kind (1: draft
+    step 1; 2: draft step 2 or the tree step; the pipelined variant has one kind)."""
+    wl = r.wl
+    if r.pipe:
+        def pipe():
+            r.ctx.block_forward(r.kv, r.toks, r.logits, r.b, r.q)
+            r.ctx.accept_pipelined(r.kv, r.logits, r.toks, r.pnver, r.b, r.q, r.acc, r.out,
+                                   temperature=wl["temperature"], top_p=wl["top_p"], seed=1234, top_k=wl["top_k"])
+        return {1: pipe}
+
+    def step1():
+        r.ctx.block_forward(r.kv, r.toks, r.logits, r.b, r.q)
+        r.accept(0)
+
+    def step2():
+        if r.tree:
+            r.forward_accept_tree()
+        else:
+            r.ctx.block_forward(r.kv, r.toks, r.logits, r.b, r.q)
+            r.accept(r.k)
+    return {1: step1, 2: step2}
+
+
+def graph_calls(r, calls):
+    """The same calls as CUDA graphs (one replay per step), or the eager calls if capture fails."""
+    torch = r.torch
+    try:
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            for f in calls.values():
+                f()
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        out = {}
+        for key, f in calls.items():
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            out[key] = g.replay
+        torch.cuda.synchronize()
+        return out, "CUDA graph of the step's C-ABI calls"
+    except Exception as e:  # graphs are an optimisation; the eager calls run the same kernels
+        print("note: e2e graph capture failed (%s); eager calls" % e, file=sys.stderr)
+        torch.cuda.synchronize()
+        return calls, "eager C-ABI calls"
+
+
 def run_e2e(r, steps, steps_per_gen):
     """The decode loop a host program writes against the C ABI: every step the host builds
     the block input from the previous step's emitted tokens (pinned buffer -> device copy),
-    calls block_forward and accept (a tree step: the tree forward and tree accept), copies the
-    emitted tokens and accepted lengths back and reads them before the next step."""
+    runs the step's calls (block_forward and accept; a tree step: the tree forward and tree
+    accept) as one CUDA-graph replay, copies the emitted tokens and accepted lengths back and
+    reads them before the next step."""
     import torch
     b, k = r.b, r.k
     qm = r.qmax
@@ -634,6 +684,7 @@ def run_e2e(r, steps, steps_per_gen):
     acc_h = torch.zeros(b, dtype=torch.int32).pin_memory()
     table = r.table.cpu()
     adaptive = [r.shape.adaptive_id] * k
+    fns, how = graph_calls(r, step_calls(r))
     r.reset()
     torch.cuda.synchronize()
 
@@ -645,7 +696,7 @@ def run_e2e(r, steps, steps_per_gen):
     h2d = d2h = 0
     st = torch.cuda.current_stream()
     if r.pipe:
-        return run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start)
+        return run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start, fns[1], how)
     t0 = time.perf_counter()
     for i in range(steps):
         j = i % steps_per_gen
@@ -663,11 +714,7 @@ def run_e2e(r, steps, steps_per_gen):
                                            for jj in range(1, k + 1)]
         tok_h[:b * q].copy_(torch.tensor(blk, dtype=torch.int32))
         r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
-        if mode == 2 and r.tree:
-            r.forward_accept_tree()
-        else:
-            r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
-            r.accept(0 if mode == 1 else k)
+        fns[mode]()
         out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
         acc_h.copy_(r.acc, non_blocking=True)
         st.synchronize()
@@ -682,10 +729,10 @@ def run_e2e(r, steps, steps_per_gen):
         d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
     return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d / steps, 1),
-            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": "eager C-ABI calls, host sync each step"}
+            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": how + ", host sync each step"}
 
 
-def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start):
+def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start, fn, how):
     """run_e2e for the pipelined variant: the host keeps each sequence's block mode, builds
     [x_0, drafts or adaptive ids, adaptive ids] and copies the per-sequence verify counts in."""
     import torch
@@ -713,10 +760,7 @@ def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adapt
         nv_h.copy_(torch.tensor(nv, dtype=torch.int32))
         r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
         r.pnver.copy_(nv_h, non_blocking=True)
-        r.ctx.block_forward(r.kv, r.toks, r.logits, b, q)
-        wl = r.wl
-        r.ctx.accept_pipelined(r.kv, r.logits, r.toks, r.pnver, b, q, r.acc, r.out, temperature=wl["temperature"],
-                               top_p=wl["top_p"], seed=1234, top_k=wl["top_k"])
+        fn()
         out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
         acc_h.copy_(r.acc, non_blocking=True)
         st.synchronize()
@@ -730,7 +774,7 @@ def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adapt
         d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
     return {"value": round(tokens / (t1 - t0), 2), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d / steps, 1),
-            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": "eager C-ABI calls, host sync each step"}
+            "d2h_bytes_per_step": round(d2h / steps, 1), "launch": how + ", host sync each step"}
 
 
 # ----------------------------------------------------------------------------- CPU oracle
