@@ -17,7 +17,7 @@
 // Epilogues: store (q, k, v before RoPE), residual add (O and down projections), and
 // SiLU(gate) * up written as the down projection's bf16 hi + lo operand.  RMSNorm and
 // RoPE + the KV append are small row kernels here (the decode path folds them into the
-// GEMMs); attention is the decode kernel in its query-group mode.
+// GEMMs); attention is the causal flash-attention kernel at the end of attention.cu.
 #include <algorithm>
 
 #include "common.cuh"
