@@ -1038,6 +1038,33 @@ def run_sweep(args):
                               "note": "x enters as bf16 hi + lo: the tensor cores execute 2 x 2MNK; includes "
                                       "the fp32 -> bf16 hi/lo operand split kernel"})
             del w
+        # a whole prefill at 7B layer dimensions (two layers, so that a profiler capture holds
+        # under a GB): per-kernel device time, and the causal attention's rate
+        sh7 = synth.SHAPES["7b"]
+        sh = synth.ModelShape("7b-2layers", 2, sh7.d_model, sh7.n_heads, sh7.head_dim, sh7.ffn_dim, sh7.vocab,
+                              sh7.adaptive_id)
+        n = args.ctx if args.ctx else 2047
+        wts = synth.make_model(sh, seed=0, device="cuda")
+        pctx = sd.Context(sh, wts, max_position=n + 64)
+        kv = pctx.kv(1, n + 16)
+        prompt = synth.prompt_ids(0, 0, n, sh.adaptive_id).cuda()
+        zero = torch.zeros(1, dtype=torch.int32, device="cuda")
+        for _ in range(2):
+            pctx.kv_commit(kv, zero, 1)
+            pctx.prefill(kv, 0, prompt)
+        torch.cuda.synchronize()
+        pctx.kv_commit(kv, zero, 1)
+        pctx.profile_begin(4096)
+        pctx.prefill(kv, 0, prompt)
+        st = pctx.profile_end()
+        att = st.get("prefill_attention", (0, 0.0))
+        att_flops = sh.n_layers * 2.0 * 2.0 * (n * n / 2.0) * sh.n_heads * sh.head_dim
+        cases.append({"kernel": "prefill_step", "shape": sh.name, "positions": n,
+                      "kernels_ms": {k: round(v[1], 4) for k, v in st.items()},
+                      "attention_TFLOP/s": round(att_flops / (att[1] / 1e3) / 1e12, 1) if att[1] else None,
+                      "note": "launches timed one by one (CUDA events); attention FLOPs 4 x n^2/2 x H x hd per "
+                              "layer (causal), algorithmic"})
+        del pctx, kv, wts
     for c in cases:
         print(json.dumps(c), flush=True)
 
