@@ -288,7 +288,7 @@ __device__ __forceinline__ int nth_id(const uint32_t (&W)[ACC_EPT], int base, co
 // threshold), those elements are copied in ascending id order into shared memory and one
 // warp runs the same selection on them: searches cost O(list / 32) per step and no block
 // barrier.  Otherwise the block-wide searches over all ids run.
-constexpr int NUC_LIST_MAX = 2048;
+constexpr int NUC_LIST_MAX = 4096;
 constexpr int NUC_FLOORS = 7;
 // floor f: 2^24 (the largest weight), 2^22, 2^20, 2^18, 2^16 (ratio 2^-8), 2^8 (2^-16), then 1
 // (every non-zero weight).  Weights of bucket b (nuc_bucket) are >= the floors f >= b.
@@ -307,7 +307,7 @@ struct NucList {
   int pick;
 };
 
-// warp-wide sums: per-lane values below 2^31 (counts, or weights of <= 64 list elements)
+// warp-wide sums: per-lane values below 2^32 (counts, or weights of <= 128 list elements)
 __device__ __forceinline__ uint64_t warp_sum_w(uint32_t v) {
   const uint32_t hi = __reduce_add_sync(0xffffffffu, v >> 16), lo = __reduce_add_sync(0xffffffffu, v & 0xFFFFu);
   return ((uint64_t)hi << 16) + lo;

@@ -276,7 +276,7 @@ def _nucleus_rows(V):
     peaked = torch.full((V,), -100.0)                                # three non-zero weights
     peaked[[7, 300, 301]] = torch.tensor([0.0, -0.5, -0.5])
     rows.append(peaked)
-    for n in (2048, 2049):                                           # list capacity, and one past it
+    for n in (4096, 4097):                                           # list capacity, and one past it
         r = torch.full((V,), -100.0)
         r[torch.arange(n) * (V // n)] = 0.0
         rows.append(r)
