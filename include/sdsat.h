@@ -369,6 +369,13 @@ SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, co
  * layer.  For tests that check a forward stage by stage.  Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_debug_workspace(sdsat_ctx* ctx, int which, int rows, float* dst_dev);
 
+/* Test hook for failure detection: one kernel waits on a barrier that nothing
+ * completes, through the bounded wait every kernel of the library uses.  After its
+ * limit (2 s) it sets device bit TIMEOUT and returns; nothing faults and the
+ * context stays usable.  Asynchronous (read the bit with sdsat_get_error).
+ * Errors: EINVAL (null ctx), ECUDA. */
+SDSAT_API sdsat_status sdsat_debug_wait_timeout(sdsat_ctx* ctx);
+
 /* out[i] = the nucleus sampler's exp (see sdsat_accept_nucleus) of in[i] <= 0. */
 SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* out_dev, int n);
 

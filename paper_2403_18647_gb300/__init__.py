@@ -99,6 +99,7 @@ def _lib():
             "sdsat_op_attention": [P, P, P, P, P, I, I, I, I, I, P],
             "sdsat_op_exp": [P, P, P, I],
             "sdsat_debug_workspace": [P, I, I, P],
+            "sdsat_debug_wait_timeout": [P],
         }
         for name, args in sig.items():
             fn = getattr(lib, name)
@@ -379,6 +380,11 @@ class Context:
         self._bind_stream()
         _check(_lib().sdsat_debug_workspace(self.handle, which, rows, _ptr(out)), "sdsat_debug_workspace")
         return out
+
+    def debug_wait_timeout(self):
+        """Queue a kernel whose bounded wait runs out (device bit TIMEOUT after ~2 s)."""
+        self._bind_stream()
+        _check(_lib().sdsat_debug_wait_timeout(self.handle), "sdsat_debug_wait_timeout")
 
     def op_exp(self, x, y):
         self._bind_stream()

@@ -962,6 +962,29 @@ cudaError_t launch_tree_compact(const int* ws, int nb, int L, int H, int hd, int
   return cudaLaunchKernelEx(&cfg, tree_compact_kernel, ws, H, hd, cap, batch, k, v);
 }
 
+// ---- the bounded wait, run out on purpose (a test hook) ----------------------------------
+// One CTA waits on an mbarrier that nothing arrives on, through the same bounded wait every
+// kernel uses: after WAIT_LIMIT_NS it sets ERR_TIMEOUT and returns; nothing faults.
+__global__ void wait_timeout_kernel(uint32_t* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  mbar_wait_bounded(&bar, 0, &abort_flag, err);
+}
+
+cudaError_t launch_wait_timeout(uint32_t* err, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1);
+  cfg.blockDim = dim3(32);
+  cfg.stream = st;
+  return cudaLaunchKernelEx(&cfg, wait_timeout_kernel, err);
+}
+
 // ---- explicit commit / rollback, and prefill commit --------------------------------------
 __global__ void commit_kernel(int* len, const int* new_len, int nb, int cap, uint32_t* err) {
   pdl_wait();
@@ -1003,8 +1026,11 @@ __global__ void exp_kernel(const float* in, float* out, int n) {
 }
 
 cudaError_t launch_exp(const float* in, float* out, int n, cudaStream_t st) {
-  exp_kernel<<<(n + 255) / 256, 256, 0, st>>>(in, out, n);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((n + 255) / 256);
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  return cudaLaunchKernelEx(&cfg, exp_kernel, in, out, n);
 }
 
 }  // namespace sdsat

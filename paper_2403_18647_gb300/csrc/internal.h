@@ -244,5 +244,7 @@ cudaError_t launch_commit(int* len, const int* new_len, int nb, int cap, uint32_
                           bool pdl);
 cudaError_t launch_add_len(int* len, int seq, int n, int cap, uint32_t* err, cudaStream_t st, bool pdl);
 cudaError_t launch_exp(const float* in, float* out, int n, cudaStream_t st);
+// a bounded wait that nothing satisfies: sets ERR_TIMEOUT after WAIT_LIMIT_NS (test hook)
+cudaError_t launch_wait_timeout(uint32_t* err, cudaStream_t st);
 
 }  // namespace sdsat

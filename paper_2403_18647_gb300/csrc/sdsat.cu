@@ -198,7 +198,10 @@ cudaError_t timed(sdsat_ctx* c, int cls, F&& launch) {
 template <typename T>
 bool dalloc(sdsat_ctx* c, T** p, size_t count) {
   void* q = nullptr;
-  if (cudaMalloc(&q, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) return false;
+  if (cudaMalloc(&q, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) {
+    cudaGetLastError();   // clear the runtime's record of the failed allocation (not sticky)
+    return false;
+  }
   if (cudaMemset(q, 0, std::max<size_t>(count, 1) * sizeof(T)) != cudaSuccess) {
     cudaFree(q);
     return false;
@@ -709,6 +712,7 @@ sdsat_status sdsat_kv_create(sdsat_ctx* c, int batch, int max_len, sdsat_kv** ou
   void *k = nullptr, *v = nullptr, *len = nullptr, *em = nullptr;
   if (cudaMalloc(&k, n * 2) != cudaSuccess || cudaMalloc(&v, n * 2) != cudaSuccess ||
       cudaMalloc(&len, batch * sizeof(int)) != cudaSuccess || cudaMalloc(&em, batch * sizeof(long long)) != cudaSuccess) {
+    cudaGetLastError();   // clear the runtime's record of the failed allocation (not sticky)
     cudaFree(k);
     cudaFree(v);
     cudaFree(len);
@@ -1031,6 +1035,11 @@ sdsat_status sdsat_build_pipelined_block(sdsat_ctx* c, sdsat_kv* kv, const int32
   return timed(c, K_BUILD_BLOCK, [&] { return launch_build_block(bp, c->stream, c->pdl); }) == cudaSuccess
              ? SDSAT_OK
              : SDSAT_ECUDA;
+}
+
+sdsat_status sdsat_debug_wait_timeout(sdsat_ctx* c) {
+  if (!c) return SDSAT_EINVAL;
+  return launch_wait_timeout(c->err, c->stream) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
 }
 
 sdsat_status sdsat_get_error(sdsat_ctx* c, uint32_t* flags) {
