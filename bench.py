@@ -212,7 +212,8 @@ class Runner:
         self.new = wl["new"]
         self.cap = self.P + 2 * self.new + 8 * self.qmax
         self.dev = device
-        self.weights = weights if weights is not None else synth.make_model(self.shape, seed=0, device=device)
+        self.weights = weights if weights is not None else synth.make_model(self.shape, seed=wl.get("seed", 0),
+                                                                            device=device)
         torch.cuda.synchronize()
         self.ctx = sd.Context(self.shape, self.weights, max_position=self.cap + 64)
         self.kv = self.ctx.kv(self.b, self.cap)
@@ -562,7 +563,7 @@ def run_ours(args, wl, rank, world):
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed 0)",
+        "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed %d)" % wl.get("seed", 0),
                    "global_batch": r.b * world, "seq_len": r.P, "new_tokens": r.new, "k": r.k, "q": r.q,
                    "draft_stub_match": branch_matches(wl) if r.tree else wl["match"],
                    "temperature": wl["temperature"], "top_p": wl["top_p"], "top_k": wl["top_k"],
@@ -892,7 +893,7 @@ def run_reference(args, wl, rank, world):
     return {"metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(t_step * 1e3, 2), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed 0)",
+            "config": {"workload": args.config, "model": shape.name + "-shaped random init (seed %d)" % wl.get("seed", 0),
                        "global_batch": wl["batch"], "seq_len": P, "k": wl["k"]},
             "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": os.cpu_count(),
                              "kind": "oracle", "sample": sample},
@@ -1085,6 +1086,9 @@ def main():
     ap.add_argument("--reps", type=int, default=50)
     ap.add_argument("--ksweep", action="store_true", help="k-sweep of the generation loop (k = 1..13)")
     ap.add_argument("--ks", default="", help="k values for --ksweep, comma separated")
+    ap.add_argument("--k", type=int, default=None, help="adaptive tokens per block (overrides the workload's)")
+    ap.add_argument("--new-tokens", type=int, default=None, help="tokens generated per generation")
+    ap.add_argument("--seed", type=int, default=None, help="seed of the synthetic weights")
     args = ap.parse_args()
     if args.sweep:
         run_sweep(args)
@@ -1094,7 +1098,10 @@ def main():
         return
     if args.warmup < 3:
         args.warmup = 3
-    wl = WORKLOADS[args.config]
+    wl = dict(WORKLOADS[args.config])
+    for key, val in (("k", args.k), ("new", args.new_tokens), ("seed", args.seed)):
+        if val is not None:
+            wl[key] = val
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if args.impl == "reference":
