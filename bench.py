@@ -796,7 +796,7 @@ def oracle_sample(shape_name, wl, weights_gpu=None, n_layers=2, repeat=1, gen_de
         if weights_gpu is not None:
             t = weights_gpu[name] if layer < 0 else weights_gpu["layers"][layer][name]
             return t.cpu()
-        return synth.make_weight(shape, name, layer, 0, "cpu")
+        return synth.make_weight(shape, name, layer, wl.get("seed", 0), "cpu")
 
     W = OM.Weights(shape, provider=provider, cache=True)
     small = synth.ModelShape("sample", n_layers, shape.d_model, shape.n_heads, shape.head_dim, shape.ffn_dim,
@@ -862,7 +862,7 @@ def run_reference(args, wl, rank, world):
     tps = workload_tokens_per_step(wl)
     q = mean_rows(wl)
     P = wl["prompt"]
-    W = OM.Weights(shape, provider=lambda n, l: synth.make_weight(shape, n, l, 0, "cpu"), cache=True)
+    W = OM.Weights(shape, provider=lambda n, l: synth.make_weight(shape, n, l, wl.get("seed", 0), "cpu"), cache=True)
     small = synth.ModelShape("sample", 1, shape.d_model, shape.n_heads, shape.head_dim, shape.ffn_dim,
                              shape.vocab, shape.adaptive_id)
     kv = OM.KVCache(small, 1, P + q)
