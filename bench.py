@@ -192,8 +192,28 @@ def kv_bytes_per_layer_slot(shape):
 
 
 # ----------------------------------------------------------------------------- our arm
+def shard_sequences(rank, b):
+    """The sequence ids rank `rank` decodes: each rank of a replica run takes its own b
+    sequences (own prompts and draft stubs), so ranks share no data and need no collective."""
+    return [rank * b + s for s in range(b)]
+
+
+def combine_ranks(ms, tokens, world, device):
+    """Whole-job (time, tokens) of a replica run: the slowest rank's time and every rank's
+    tokens (value = tokens / time)."""
+    if world == 1:
+        return ms, tokens
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms), float(tokens)], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return mx[0].item(), t[1].item()
+
+
 class Runner:
-    def __init__(self, wl, device, weights=None):
+    def __init__(self, wl, device, weights=None, shard=0):
         import torch
         import synth
         import paper_2403_18647_gb300 as sd
@@ -225,7 +245,8 @@ class Runner:
         self.parent = torch.tensor(chains_parent(self.width, self.k) * self.b, dtype=torch.int32, device=device)
         self.pmode = torch.ones(self.b, dtype=torch.int32, device=device)    # pipelined: the previous block's mode
         self.pnver = torch.zeros(self.b, dtype=torch.int32, device=device)
-        self.prompts = [synth.prompt_ids(0, s, self.P, self.shape.adaptive_id, device) for s in range(self.b)]
+        self.seq_ids = shard_sequences(shard, self.b)
+        self.prompts = [synth.prompt_ids(0, i, self.P, self.shape.adaptive_id, device) for i in self.seq_ids]
         for s in range(self.b):
             self.ctx.prefill(self.kv, s, self.prompts[s][:-1].contiguous())
         self.prefill_ms = self._time_prefill()
@@ -296,7 +317,7 @@ class Runner:
             for s in range(self.b):
                 full = torch.zeros(self.stride, dtype=torch.int32, device=self.dev)
                 full[self.P:self.P + n_run] = ref[:n_run, s]
-                table[w, s] = self.synth.stub_table(w, s, full, match, self.shape.vocab)
+                table[w, s] = self.synth.stub_table(w, self.seq_ids[s], full, match, self.shape.vocab)
         self.table = table.contiguous()
         self.ref = ref
 
@@ -483,7 +504,7 @@ def run_ours(args, wl, rank, world):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    r = Runner(wl, dev)
+    r = Runner(wl, dev, shard=rank)
     shape = r.shape
     steps_per_gen, lens, toks_cal, flags = r.calibrate()
     # schedule the timed region as whole-generation-aligned steps
@@ -517,12 +538,7 @@ def run_ours(args, wl, rank, world):
     ms = e0.elapsed_time(e1)
     tokens = r.ctx.kv_emitted(r.kv).sum().item() - em0
     flags |= r.ctx.get_error()
-    if world > 1:
-        t = torch.tensor([ms, float(tokens)], device=dev)
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        ms, tokens = mx[0].item(), t[1].item()
+    ms, tokens = combine_ranks(ms, tokens, world, dev)
     value = tokens / (ms / 1e3)
     # --- profiled pass (per-kernel CUDA events; launches serialised) for the roofline
     r.reset()
