@@ -10,28 +10,34 @@
 // The bytes are the K and V rows (bf16, hd*2 bytes each), read once per
 // (sequence, head) for all q rows together.
 //
-// Work is split into units of ATT_UNIT = 64 consecutive slots of one
-// (sequence, head), ordered (sequence, head, unit).  One wave of P CTAs (two
-// per SM) reads the committed lengths, counts the U units and takes the
-// contiguous range [iU/P, (i+1)U/P): every CTA streams the same number of
-// K/V bytes.  One thread keeps a two-stage ring of K and V tiles (TMA, boxes
-// of 64 dims x 64 rows, 128-byte swizzle) full; tiles made of committed slots
-// only are requested before the QKV projection has finished, and the next
-// ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on the tensor
-// cores (mma.sync m16n8k16) in transposed form, so that the q <= 8 block rows
-// fill an N = 8 tile instead of padding an M = 16 one: S^T = K Q^T with each
-// warp on 16 keys, an online-softmax update of the running row max and
-// exp-sum (reductions over the warp's lanes, then the warps via shared
+// Work: the grid is nclusters thread-block clusters of cs CTAs, all resident
+// at once (launch_attention picks the largest cs <= ATT_CS_MAX for which one
+// cluster per (sequence, head) pair fits on the GPU with room to spare; else
+// cs = 1 and each CTA takes several pairs).  Three CTAs fit on an SM for q <= 8
+// (two for q <= 16).  Cluster c takes the pairs c, c + nclusters, ...; the
+// nu units of ATT_UNIT = 64 consecutive slots of a pair are split over the
+// cluster's CTAs as [r*nu/cs, (r+1)*nu/cs) for CTA rank r.  One thread keeps a
+// two-stage ring of K and V tiles (TMA, boxes of 64 dims x 64 rows, 128-byte
+// swizzle) full, walking the CTA's units pair by pair; tiles made of committed
+// slots only are requested before the QKV projection has finished, and the
+// next ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on the
+// tensor cores (mma.sync m16n8k16) in transposed form, so that the q <= 8
+// block rows fill an N = 8 tile instead of padding an M = 16 one: S^T = K Q^T
+// with each warp on 16 keys, an online-softmax update of the running row max
+// and exp-sum (reductions over the warp's lanes, then the warps via shared
 // memory), then O^T = O^T * alpha + V^T P^T with each warp on hd/4
 // dimensions.  Q and P enter as bf16 hi + lo pairs (two MMAs each), K and V
 // are the cache's own bf16 values, accumulation is fp32.
 //
-// A CTA's run of units of one (sequence, head) ends in a partial result (row
-// max, exp-sum, unnormalised output).  The last of the <= ATT_SEG_MAX CTAs
-// sharing the pair (per-pair counter, no waiting) merges the partials in CTA
-// order with the usual log-sum-exp rescaling -- deterministic -- and writes
-// the output in fp32 and as the O projection's bf16 hi + lo operand.
+// Each CTA's run over its units of a pair ends in a partial result (row max,
+// exp-sum, unnormalised output) that it leaves in its own shared memory; after
+// a cluster barrier every CTA merges its share of the pair's output elements
+// from the cs partials through distributed shared memory, in rank order with
+// the usual log-sum-exp rescaling (deterministic), and writes them in fp32 and
+// as the O projection's bf16 hi + lo operand.  A second cluster barrier keeps
+// the partials in place until every CTA of the cluster has read them.
 #include <algorithm>
+#include <cstdlib>
 
 #include "common.cuh"
 #include "internal.h"
@@ -40,9 +46,11 @@ namespace sdsat {
 
 constexpr int ATT_STAGES = 2;
 constexpr int ATT_PREFETCH = 4;   // units past the ring requested into L2 ahead of their loads
+constexpr int ATT_SPARE_CLUSTERS = 8;   // room left for this many more clusters (measured: 7B/13B shapes, b = 1, 4)
 
-template <int HD>
+template <int HD, int QT = 2>
 struct AttCfg {
+  static constexpr int ROWS = QT * 8;                    // query rows the tiles hold
   static constexpr int HALVES = HD / 64;                 // 64-dim column boxes per row
   static constexpr int HALF_BYTES = ATT_UNIT * 128;      // one box: 64 rows x 64 dims bf16
   static constexpr int TILE = HALF_BYTES * HALVES;       // K (or V) of one unit
@@ -50,14 +58,16 @@ struct AttCfg {
   static constexpr int QSTRIDE = HD * 2 + 16;            // bytes per row of the bf16 Q tiles (padded)
   static constexpr int PSTRIDE = ATT_UNIT * 2 + 16;      // bytes per row of the bf16 P tiles (padded)
   static constexpr int RED = 17;                         // floats per row of the row-reduction scratch
+  // Q hi + lo tiles; once the CTA's units of a pair are done, its partial output [ROWS][HD] fp32
   static constexpr size_t OFF_Q = (size_t)ATT_STAGES * STAGE;
-  static constexpr size_t OFF_P = OFF_Q + 2 * 16 * QSTRIDE;
-  static constexpr size_t OFF_RED = OFF_P + 2 * 16 * PSTRIDE;                       // [16][RED]
-  static constexpr size_t OFF_MERGE = OFF_RED + 16 * RED * 4;                       // ms, ls, w [16][SEG], inv [16]
-  static constexpr size_t OFF_SEQ = OFF_MERGE + (3 * 16 * ATT_SEG_MAX + 16) * 4;    // len, units [64], first unit [65]
-  static constexpr size_t OFF_ANC = OFF_SEQ + (64 + 64 + 65) * 4;                   // [16] visible block rows per row
+  // P hi + lo tiles; once the units are done, the partial's row max and exp-sum [ROWS][2]
+  static constexpr size_t OFF_P = OFF_Q + 2 * ROWS * QSTRIDE;
+  static constexpr size_t OFF_RED = OFF_P + 2 * ROWS * PSTRIDE;                     // [16][RED]
+  static constexpr size_t OFF_SEQ = OFF_RED + 16 * RED * 4;                         // len, units [64]
+  static constexpr size_t OFF_ANC = OFF_SEQ + (64 + 64) * 4;                        // [16] visible block rows per row
   static constexpr size_t OFF_BAR = (OFF_ANC + 16 * 4 + 7) / 8 * 8;
   static constexpr size_t SMEM = 1024 + OFF_BAR + ATT_STAGES * 8 + 16;
+  static_assert(ROWS * HD * 4 <= 2 * ROWS * QSTRIDE, "the partial output fits in the Q tiles");
 };
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
@@ -84,41 +94,35 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo_elem, float hi_elem) {
          ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(hi_elem)) << 16);
 }
 
-// CTA owning unit u when U units are split over P CTAs as [iU/P, (i+1)U/P)
-__device__ __forceinline__ int att_cta_of(int u, int U, int P) {
-  return (int)(((long long)(u + 1) * P - 1) / U);
-}
-
 // QT: tiles of 8 query rows (1 for q <= 8, 2 for q <= 16)
 template <int HD, int QT>
-__global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ AttnParams p) {
-  using C = AttCfg<HD>;
+__global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const __grid_constant__ AttnParams p) {
+  using C = AttCfg<HD, QT>;
   constexpr int KSTEPS = HD / 16;          // MMA k-steps over the head dimension
   constexpr int MT = HD / 64;              // 16-dimension tiles per warp in V^T P^T
   constexpr int D4 = HD / 4;               // float4 columns of an output row
+  constexpr int QI = QT * 8 * (HD / 2) / 128;   // (row, 2 dims) items of the q tiles per thread
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* Qh = smem + C::OFF_Q;                    // bf16 [16][HD] (scaled q, hi part), padded rows
-  uint8_t* Ql = Qh + 16 * C::QSTRIDE;               // lo part
-  uint8_t* Ph = smem + C::OFF_P;                    // bf16 [16][ATT_UNIT] softmax numerators, hi part
-  uint8_t* Pl = Ph + 16 * C::PSTRIDE;
+  uint8_t* Qh = smem + C::OFF_Q;                    // bf16 [ROWS][HD] (scaled q, hi part), padded rows
+  uint8_t* Ql = Qh + C::ROWS * C::QSTRIDE;          // lo part
+  float* po = reinterpret_cast<float*>(smem + C::OFF_Q);        // [ROWS][HD] partial output (after the units)
+  uint8_t* Ph = smem + C::OFF_P;                    // bf16 [ROWS][ATT_UNIT] softmax numerators, hi part
+  uint8_t* Pl = Ph + C::ROWS * C::PSTRIDE;
+  float* pml = reinterpret_cast<float*>(smem + C::OFF_P);       // [ROWS][2] partial row max, exp-sum (after the units)
   float* red = reinterpret_cast<float*>(smem + C::OFF_RED);     // row-reduction scratch
-  float* ms = reinterpret_cast<float*>(smem + C::OFF_MERGE);    // [16][ATT_SEG_MAX] partial maxima
-  float* ls = ms + 16 * ATT_SEG_MAX;                            // partial exp-sums
-  float* wg = ls + 16 * ATT_SEG_MAX;                            // merge weights
-  float* inv = wg + 16 * ATT_SEG_MAX;                           // [16] 1 / L
   int* len_seq = reinterpret_cast<int*>(smem + C::OFF_SEQ);     // [64] committed length of each sequence
   int* nu_seq = len_seq + 64;                                   // [64] units per head of each sequence
-  int* base = nu_seq + 64;                                      // [65] first unit of each sequence
   uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + C::OFF_ANC);   // [16] block rows row j sees (bit i)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);   // [ATT_STAGES] K and V of the stage landed
   volatile int* abort_flag = reinterpret_cast<volatile int*>(full + ATT_STAGES);
-  int* s_last = reinterpret_cast<int*>(full + ATT_STAGES) + 1;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, tig = lane & 3;
   const int mi = lane >> 3, r8 = lane & 7;        // ldmatrix: this thread's matrix and row
   const int q = p.q, H = p.H;
+  const int CS = p.cs, NC = p.nclusters;
+  const int rank = (int)cluster_ctarank(), cl = (int)blockIdx.x / CS;
   const unsigned long long t_entry = p.trace.rec ? globaltimer_ns() : 0;
   pdl_trigger();
 
@@ -136,39 +140,43 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     fence_mbar_init();
   }
   __syncthreads();
-  if (tid == 0) {
-    int acc = 0;
-    for (int s = 0; s < p.nb; ++s) {
-      base[s] = acc;
-      acc += H * nu_seq[s];
-    }
-    base[p.nb] = acc;
-  }
-  __syncthreads();
-  const int U = base[p.nb];
-  const int P = min((int)gridDim.x, U);           // every CTA below P owns at least one unit
-  const int cta = blockIdx.x;
-  if (cta >= P) return;
-  const int u0 = (int)((long long)cta * U / P), u1 = (int)((long long)(cta + 1) * U / P);
-  const int n = u1 - u0;
+  const int npairs = p.nb * H;
 
-  // unit u -> (sequence sl, head h, unit c of the pair)
-  auto locate = [&](int u, int& s, int& hh, int& cc) {
-    s = 0;
-    while (base[s + 1] <= u) ++s;
-    const int r = u - base[s];
-    hh = r / nu_seq[s];
-    cc = r % nu_seq[s];
+  // this CTA's units [cb, ce) of pair pi (sequence pi / H, head pi % H)
+  auto slice = [&](int pi, int& cb, int& ce) {
+    const int nu = nu_seq[pi / H];
+    cb = nu * rank / CS;
+    ce = nu * (rank + 1) / CS;
   };
-  // first cache row of unit u, and whether all of its slots are committed
-  auto unit_row = [&](int u, bool& committed) {
-    int s, hh, cc;
-    locate(u, s, hh, cc);
-    committed = (cc + 1) * ATT_UNIT <= len_seq[s];
-    return p.row0 + ((p.seq0 + s) * H + hh) * p.cap + cc * ATT_UNIT;
+  // a position in the CTA's sequence of units: unit c of pair pi, its slice ending at ce
+  struct Cursor {
+    int pi, c, ce;
+  };
+  auto seek = [&](Cursor& u, int pi) {   // the first unit of the CTA's slices from pair pi on
+    for (; pi < npairs; pi += NC) {
+      int cb, ce;
+      slice(pi, cb, ce);
+      if (cb < ce) {
+        u.pi = pi;
+        u.c = cb;
+        u.ce = ce;
+        return;
+      }
+    }
+    u.pi = npairs;
+    u.c = u.ce = 0;
+  };
+  auto advance = [&](Cursor& u) {
+    if (++u.c == u.ce) seek(u, u.pi + NC);
+  };
+  // first cache row of the cursor's unit, and whether all of its slots are committed
+  auto unit_row = [&](const Cursor& u, bool& committed) {
+    const int s = u.pi / H, hh = u.pi - s * H;
+    committed = (u.c + 1) * ATT_UNIT <= len_seq[s];
+    return p.row0 + ((p.seq0 + s) * H + hh) * p.cap + u.c * ATT_UNIT;
   };
   uint64_t pol = 0;
-  auto issue = [&](int k, int row) {   // unit u0 + k into stage k % ATT_STAGES
+  auto issue = [&](int k, int row) {   // the CTA's unit k into stage k % ATT_STAGES
     uint8_t* st = smem + (size_t)(k % ATT_STAGES) * C::STAGE;
     uint64_t* bar = &full[k % ATT_STAGES];
     mbar_arrive_expect_tx(bar, C::STAGE);
@@ -185,7 +193,10 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
       tma_prefetch_l2_2d(&p.vmap, hh * 64, row);
     }
   };
-  int issued = 0;   // units whose loads were issued (thread 0)
+  // thread 0: units whose loads were issued, the next unit to load (isu) and the next
+  // to prefetch into L2 (pfc, ATT_PREFETCH units past the ring)
+  int issued = 0;
+  Cursor isu{npairs, 0, 0}, pfc{npairs, 0, 0};
   if (tid == 0) {
     tma_prefetch_desc(&p.kmap);
     tma_prefetch_desc(&p.vmap);
@@ -193,28 +204,34 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     // Tiles of committed slots do not depend on the QKV projection: the first ones go
     // to the ring now, the next ATT_PREFETCH into L2 (and one more each time the ring is
     // refilled), so that the ring's loads are L2 hits instead of HBM round trips.
-    for (; issued < min(n, ATT_STAGES); ++issued) {
+    seek(isu, cl);
+    for (; issued < ATT_STAGES && isu.pi < npairs; ++issued) {
       bool committed;
-      const int row = unit_row(u0 + issued, committed);
+      const int row = unit_row(isu, committed);
       if (!committed) break;
       issue(issued, row);
+      advance(isu);
     }
-    for (int k = ATT_STAGES; k < min(n, ATT_STAGES + ATT_PREFETCH); ++k) {
+    pfc = isu;
+    for (int k = issued; k < ATT_STAGES && pfc.pi < npairs; ++k) advance(pfc);
+    for (int k = 0; k < ATT_PREFETCH && pfc.pi < npairs; ++k) {
       bool committed;
-      const int row = unit_row(u0 + k, committed);
+      const int row = unit_row(pfc, committed);
       if (committed) prefetch(row);
+      advance(pfc);
     }
   }
   pdl_wait();   // q and this forward's new K/V rows come from the QKV projection
   const unsigned long long t_wait = p.trace.rec ? globaltimer_ns() : 0;
   if (tid == 0) {
-    for (; issued < min(n, ATT_STAGES); ++issued) {
+    for (; issued < ATT_STAGES && isu.pi < npairs; ++issued) {
       bool committed;
-      issue(issued, unit_row(u0 + issued, committed));
+      issue(issued, unit_row(isu, committed));
+      advance(isu);
     }
   }
   unsigned long long t_k = 0, t_part = 0, t_merge = 0;
-  unsigned merges = 0;
+  unsigned pairs_done = 0;
 
   const float scale = rsqrtf((float)HD);
   const int kb = warp * 16;                       // first key (within the unit) of this warp's scores
@@ -224,323 +241,274 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
   // t*8 + 2*tig + {0, 1} and keeps their running max and exp-sum in registers
   float O[MT][QT][4], Ol[MT][QT][4];
   float mr[QT][2], lr[QT][2];
+  int k = 0;                                      // units of this CTA consumed (ring position)
+  for (int pi = cl; pi < npairs; pi += NC) {
+    const int sl = pi / H, h = pi - sl * H;
+    int cb, ce;
+    slice(pi, cb, ce);
 #pragma unroll
-  for (int t = 0; t < QT; ++t) mr[t][0] = mr[t][1] = -INFINITY, lr[t][0] = lr[t][1] = 0.f;
-  int sl = 0, h = 0, c = 0;
-  locate(u0, sl, h, c);
-  int seg_first = u0;                             // first unit of the current (sequence, head) run
-  for (int k = 0; k < n; ++k) {
-    const int u = u0 + k;
-    if (u == seg_first) {
-      // ---- a new (sequence, head): the rows' visible block rows (causal: 0..j; tree: the
-      // ancestors and the row itself), q (scaled by 1/sqrt(hd)) as bf16 hi + lo, rows >= q zero
+    for (int t = 0; t < QT; ++t) mr[t][0] = mr[t][1] = -INFINITY, lr[t][0] = lr[t][1] = 0.f;
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+      for (int t = 0; t < QT; ++t)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) O[mt][t][e] = Ol[mt][t][e] = 0.f;
+    if (cb < ce) {
+      // ---- the rows' visible block rows (causal: 0..j; tree: the ancestors and the row
+      // itself), q (scaled by 1/sqrt(hd)) as bf16 hi + lo, rows >= q zero; every load first
       if (tid < 16) anc_s[tid] = (p.anc && tid < q) ? __ldcg(p.anc + sl * q + tid) : (2u << tid) - 1u;
-      for (int i = tid; i < 16 * (HD / 2); i += 128) {
-        const int j = i / (HD / 2), d = (i % (HD / 2)) * 2;
-        float x0 = 0.f, x1 = 0.f;
-        if (j < q) {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(p.Q + (size_t)(sl * q + j) * p.q_ld + h * HD + d));
-          x0 = v.x * scale;
-          x1 = v.y * scale;
-        }
+      float2 qv[QI];
+#pragma unroll
+      for (int r = 0; r < QI; ++r) {
+        const int i = tid + 128 * r, j = i / (HD / 2), d = (i % (HD / 2)) * 2;
+        qv[r] = j < q ? __ldcg(reinterpret_cast<const float2*>(p.Q + (size_t)(sl * q + j) * p.q_ld + h * HD + d))
+                      : make_float2(0.f, 0.f);
+      }
+#pragma unroll
+      for (int r = 0; r < QI; ++r) {
+        const int i = tid + 128 * r, j = i / (HD / 2), d = (i % (HD / 2)) * 2;
+        const float x0 = qv[r].x * scale, x1 = qv[r].y * scale;
         const __nv_bfloat16 h0 = __float2bfloat16_rn(x0), h1 = __float2bfloat16_rn(x1);
         *reinterpret_cast<uint32_t*>(Qh + j * C::QSTRIDE + d * 2) =
             (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
         *reinterpret_cast<uint32_t*>(Ql + j * C::QSTRIDE + d * 2) =
             pack_bf16(x0 - __bfloat162float(h0), x1 - __bfloat162float(h1));
       }
-#pragma unroll
-      for (int t = 0; t < QT; ++t) mr[t][0] = mr[t][1] = -INFINITY, lr[t][0] = lr[t][1] = 0.f;
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt)
-#pragma unroll
-        for (int t = 0; t < QT; ++t)
-#pragma unroll
-          for (int e = 0; e < 4; ++e) O[mt][t][e] = Ol[mt][t][e] = 0.f;
       __syncthreads();
     }
     const int len = len_seq[sl];
     const int nkeys = min(len + q, p.cap);
-    const int c0 = c * ATT_UNIT;                  // slot of the unit's first key
-    const uint8_t* Kt = smem + (size_t)(k % ATT_STAGES) * C::STAGE;
-    const uint8_t* Vt = Kt + C::TILE;
-    const bool ok = mbar_wait_bounded(&full[k % ATT_STAGES], (k / ATT_STAGES) & 1, abort_flag, p.err);
-    __syncwarp();   // lanes leave the polling loop at different times: reconverge
-    if (k == 0 && p.trace.rec) t_k = globaltimer_ns();
+    for (int c = cb; c < ce; ++c, ++k) {
+      const int c0 = c * ATT_UNIT;                  // slot of the unit's first key
+      const uint8_t* Kt = smem + (size_t)(k % ATT_STAGES) * C::STAGE;
+      const uint8_t* Vt = Kt + C::TILE;
+      const bool ok = mbar_wait_bounded(&full[k % ATT_STAGES], (k / ATT_STAGES) & 1, abort_flag, p.err);
+      __syncwarp();   // lanes leave the polling loop at different times: reconverge
+      if (k == 0 && p.trace.rec) t_k = globaltimer_ns();
 
-    // ---- S^T = K Q^T for this warp's 16 keys: m16n8k16 with A = K (16 keys x 16 dims) and
-    // B = Q^T (16 dims x 8 query rows), so up to 8 block rows fill one N = 8 tile
-    float St[QT][4], Sl[QT][4];   // products with the hi and the lo part of q
-#pragma unroll
-    for (int t = 0; t < QT; ++t)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) St[t][e] = Sl[t][e] = 0.f;
-    if (ok) {
-#pragma unroll
-      for (int kk = 0; kk < KSTEPS; ++kk) {
-        const int hh = kk >> 2, cg = 2 * (kk & 3);  // 64-dim half and first 16-byte granule
-        const int key = kb + r8 + 8 * (mi & 1), cc = cg + (mi >> 1);
-        uint32_t a0, a1, a2, a3;
-        ldsm_x4(smem_u32(Kt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), a0, a1, a2, a3);
-#pragma unroll
-        for (int t = 0; t < QT; ++t) {
-          uint32_t bh0, bh1, bl0, bl1;   // q rows t*8 .. t*8+7: hi (matrices 0, 1), lo (2, 3)
-          const uint8_t* qsrc = (mi >> 1) ? Ql : Qh;
-          ldsm_x4(smem_u32(qsrc + (t * 8 + r8) * C::QSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), bh0, bh1, bl0, bl1);
-          mma_bf16_16816(St[t], a0, a1, a2, a3, bh0, bh1);
-          mma_bf16_16816(Sl[t], a0, a1, a2, a3, bl0, bl1);
-        }
-      }
+      // ---- S^T = K Q^T for this warp's 16 keys: m16n8k16 with A = K (16 keys x 16 dims) and
+      // B = Q^T (16 dims x 8 query rows), so up to 8 block rows fill one N = 8 tile
+      float St[QT][4], Sl[QT][4];   // products with the hi and the lo part of q
 #pragma unroll
       for (int t = 0; t < QT; ++t)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) St[t][e] += Sl[t][e];
-    }
-    // St[t][e] is the score of key kb + g + 8*(e >> 1) for query row t*8 + 2*tig + (e & 1).
-    // mask: row j sees key slot kp iff kp < len, or kp = len + i for a block row i that
-    // anc_s[j] marks (and kp < nkeys, j < q)
+        for (int e = 0; e < 4; ++e) St[t][e] = Sl[t][e] = 0.f;
+      if (ok) {
 #pragma unroll
-    for (int t = 0; t < QT; ++t)
+        for (int kk = 0; kk < KSTEPS; ++kk) {
+          const int hh = kk >> 2, cg = 2 * (kk & 3);  // 64-dim half and first 16-byte granule
+          const int key = kb + r8 + 8 * (mi & 1), cc = cg + (mi >> 1);
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(smem_u32(Kt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), a0, a1, a2, a3);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int j = t * 8 + 2 * tig + (e & 1);
-        const int kp = c0 + kb + g + 8 * (e >> 1);
-        if (!ok || j >= q || kp >= nkeys || (kp >= len && !((anc_s[j] >> (kp - len)) & 1u))) St[t][e] = -INFINITY;
+          for (int t = 0; t < QT; ++t) {
+            uint32_t bh0, bh1, bl0, bl1;   // q rows t*8 .. t*8+7: hi (matrices 0, 1), lo (2, 3)
+            const uint8_t* qsrc = (mi >> 1) ? Ql : Qh;
+            ldsm_x4(smem_u32(qsrc + (t * 8 + r8) * C::QSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), bh0, bh1, bl0, bl1);
+            mma_bf16_16816(St[t], a0, a1, a2, a3, bh0, bh1);
+            mma_bf16_16816(Sl[t], a0, a1, a2, a3, bl0, bl1);
+          }
+        }
+#pragma unroll
+        for (int t = 0; t < QT; ++t)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) St[t][e] += Sl[t][e];
       }
-    // ---- the unit's row maxima: over the warp's lanes holding other keys (g), then the four
-    // warps through shared memory; the running statistics stay in registers
-    float* redm = red;          // [4 warps][16 rows] unit row maxima
-    float* redl = red + 64;     // [4 warps][16 rows] unit row exp-sums
-    float mx[QT][2];
-#pragma unroll
-    for (int t = 0; t < QT; ++t) {
-      mx[t][0] = fmaxf(St[t][0], St[t][2]);
-      mx[t][1] = fmaxf(St[t][1], St[t][3]);
-#pragma unroll
-      for (int o = 4; o < 32; o <<= 1) {
-        mx[t][0] = fmaxf(mx[t][0], __shfl_xor_sync(0xffffffffu, mx[t][0], o));
-        mx[t][1] = fmaxf(mx[t][1], __shfl_xor_sync(0xffffffffu, mx[t][1], o));
-      }
-      if (g == 0) {
-        redm[warp * 16 + t * 8 + 2 * tig] = mx[t][0];
-        redm[warp * 16 + t * 8 + 2 * tig + 1] = mx[t][1];
-      }
-    }
-    __syncthreads();
-    float al[QT][2];   // rescale of what the units before contributed
-#pragma unroll
-    for (int t = 0; t < QT; ++t)
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int j = t * 8 + 2 * tig + i;
-        const float mc = fmaxf(fmaxf(redm[j], redm[16 + j]), fmaxf(redm[32 + j], redm[48 + j]));
-        const float mn = fmaxf(mr[t][i], mc);
-        al[t][i] = (mn == -INFINITY) ? 1.f : __expf(mr[t][i] - mn);
-        mr[t][i] = mn;
-      }
-    // ---- P^T = exp(S^T - m) as bf16 hi + lo, stored as P [query row][key], and its row sums
-    float rs[QT][2];   // this thread's part of the unit row sums
-#pragma unroll
-    for (int t = 0; t < QT; ++t) {
-      rs[t][0] = rs[t][1] = 0.f;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int i = e & 1, j = t * 8 + 2 * tig + i, key = kb + g + 8 * (e >> 1);
-        const float pv = (St[t][e] == -INFINITY) ? 0.f : __expf(St[t][e] - mr[t][i]);
-        rs[t][i] += pv;
-        const __nv_bfloat16 hi = __float2bfloat16_rn(pv);
-        *reinterpret_cast<__nv_bfloat16*>(Ph + j * C::PSTRIDE + key * 2) = hi;
-        *reinterpret_cast<__nv_bfloat16*>(Pl + j * C::PSTRIDE + key * 2) = __float2bfloat16_rn(pv - __bfloat162float(hi));
-      }
-#pragma unroll
-      for (int o = 4; o < 32; o <<= 1) {
-        rs[t][0] += __shfl_xor_sync(0xffffffffu, rs[t][0], o);
-        rs[t][1] += __shfl_xor_sync(0xffffffffu, rs[t][1], o);
-      }
-      if (g == 0) {
-        redl[warp * 16 + t * 8 + 2 * tig] = rs[t][0];
-        redl[warp * 16 + t * 8 + 2 * tig + 1] = rs[t][1];
-      }
-    }
-    __syncthreads();   // P tiles and the row sums are complete
-#pragma unroll
-    for (int t = 0; t < QT; ++t)
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int j = t * 8 + 2 * tig + i;
-        lr[t][i] = lr[t][i] * al[t][i] + ((redl[j] + redl[16 + j]) + (redl[32 + j] + redl[48 + j]));
-      }
-    // ---- O^T = O^T * alpha + V^T P^T: A = V^T (16 dims x 16 keys, transposed loads of the V
-    // tile), B = P^T (16 keys x 8 query rows), for this warp's dimensions and every query tile
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
+      // St[t][e] is the score of key kb + g + 8*(e >> 1) for query row t*8 + 2*tig + (e & 1).
+      // mask: row j sees key slot kp iff kp < len, or kp = len + i for a block row i that
+      // anc_s[j] marks (and kp < nkeys, j < q)
 #pragma unroll
       for (int t = 0; t < QT; ++t)
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          O[mt][t][e] *= al[t][e & 1];
-          Ol[mt][t][e] *= al[t][e & 1];
+          const int j = t * 8 + 2 * tig + (e & 1);
+          const int kp = c0 + kb + g + 8 * (e >> 1);
+          if (!ok || j >= q || kp >= nkeys || (kp >= len && !((anc_s[j] >> (kp - len)) & 1u))) St[t][e] = -INFINITY;
         }
-    if (ok) {
+      // ---- the unit's row maxima: over the warp's lanes holding other keys (g), then the four
+      // warps through shared memory; the running statistics stay in registers
+      float* redm = red;          // [4 warps][16 rows] unit row maxima
+      float* redl = red + 64;     // [4 warps][16 rows] unit row exp-sums
+      float mx[QT][2];
 #pragma unroll
-      for (int kk = 0; kk < ATT_UNIT / 16; ++kk) {
-        uint32_t va[MT][4];
+      for (int t = 0; t < QT; ++t) {
+        mx[t][0] = fmaxf(St[t][0], St[t][2]);
+        mx[t][1] = fmaxf(St[t][1], St[t][3]);
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-          const int key = kk * 16 + r8 + 8 * (mi >> 1);
-          const int dim = db + 16 * mt + 8 * (mi & 1);
-          const int hh = dim >> 6, cc = (dim & 63) >> 3;
-          ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), va[mt][0], va[mt][1],
-                    va[mt][2], va[mt][3]);
+        for (int o = 4; o < 32; o <<= 1) {
+          mx[t][0] = fmaxf(mx[t][0], __shfl_xor_sync(0xffffffffu, mx[t][0], o));
+          mx[t][1] = fmaxf(mx[t][1], __shfl_xor_sync(0xffffffffu, mx[t][1], o));
         }
-#pragma unroll
-        for (int t = 0; t < QT; ++t) {
-          uint32_t ph0, ph1, pl0, pl1;   // P rows t*8 .. t*8+7, keys kk*16 ..: hi (0, 1), lo (2, 3)
-          const uint8_t* psrc = (mi >> 1) ? Pl : Ph;
-          ldsm_x4(smem_u32(psrc + (t * 8 + r8) * C::PSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), ph0, ph1, pl0, pl1);
-#pragma unroll
-          for (int mt = 0; mt < MT; ++mt) {
-            mma_bf16_16816(O[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], ph0, ph1);
-            mma_bf16_16816(Ol[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], pl0, pl1);
-          }
+        if (g == 0) {
+          redm[warp * 16 + t * 8 + 2 * tig] = mx[t][0];
+          redm[warp * 16 + t * 8 + 2 * tig + 1] = mx[t][1];
         }
       }
-    }
-    __syncthreads();   // the stage, P and the row statistics are consumed
-    if (tid == 0 && issued < n && !*abort_flag) {   // refill the freed stage, extend the L2 window
-      bool committed;
-      issue(issued, unit_row(u0 + issued, committed));
-      if (issued + ATT_PREFETCH < n) prefetch(unit_row(u0 + issued + ATT_PREFETCH, committed));
-      ++issued;
-    }
-
-    // ---- end of this CTA's run of units of the pair: publish the partial result
-    const int nu = nu_seq[sl];
-    if (k == n - 1 || c == nu - 1) {
-      const int hu0 = base[sl] + h * nu;                       // the pair's units [hu0, hu0 + nu)
-      const int j0 = att_cta_of(hu0, U, P), j1 = att_cta_of(hu0 + nu - 1, U, P);
-      const int slot = cta - j0, nseg = j1 - j0 + 1;           // <= (nu-1)P/U + 2 <= P/H + 2 <= ATT_SEG_MAX
-      const size_t pair = (size_t)h * ATT_SEG_MAX;
-      const bool fits = nseg <= ATT_SEG_MAX;                   // always, for grids launch_attention makes
-      if (!fits && tid == 0) set_error(p.err, ERR_CAPACITY);
-      if (warp == 0 && g == 0 && fits) {   // the statistics of this thread's query rows
+      __syncthreads();
+      float al[QT][2];   // rescale of what the units before contributed
 #pragma unroll
-        for (int t = 0; t < QT; ++t)
+      for (int t = 0; t < QT; ++t)
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            const int j = t * 8 + 2 * tig + i;
-            if (j < q) {
-              float* ml = p.part_ml + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * 2;
-              ml[0] = mr[t][i];
-              ml[1] = lr[t][i];
-            }
-          }
+        for (int i = 0; i < 2; ++i) {
+          const int j = t * 8 + 2 * tig + i;
+          const float mc = fmaxf(fmaxf(redm[j], redm[16 + j]), fmaxf(redm[32 + j], redm[48 + j]));
+          const float mn = fmaxf(mr[t][i], mc);
+          al[t][i] = (mn == -INFINITY) ? 1.f : __expf(mr[t][i] - mn);
+          mr[t][i] = mn;
+        }
+      // ---- P^T = exp(S^T - m) as bf16 hi + lo, stored as P [query row][key], and its row sums
+      float rs[QT][2];   // this thread's part of the unit row sums
+#pragma unroll
+      for (int t = 0; t < QT; ++t) {
+        rs[t][0] = rs[t][1] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int i = e & 1, j = t * 8 + 2 * tig + i, key = kb + g + 8 * (e >> 1);
+          const float pv = (St[t][e] == -INFINITY) ? 0.f : __expf(St[t][e] - mr[t][i]);
+          rs[t][i] += pv;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(pv);
+          *reinterpret_cast<__nv_bfloat16*>(Ph + j * C::PSTRIDE + key * 2) = hi;
+          *reinterpret_cast<__nv_bfloat16*>(Pl + j * C::PSTRIDE + key * 2) = __float2bfloat16_rn(pv - __bfloat162float(hi));
+        }
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+          rs[t][0] += __shfl_xor_sync(0xffffffffu, rs[t][0], o);
+          rs[t][1] += __shfl_xor_sync(0xffffffffu, rs[t][1], o);
+        }
+        if (g == 0) {
+          redl[warp * 16 + t * 8 + 2 * tig] = rs[t][0];
+          redl[warp * 16 + t * 8 + 2 * tig + 1] = rs[t][1];
+        }
       }
-      // O^T[mt][t][e] is dimension db + 16*mt + g + 8*(e >> 1) of query row t*8 + 2*tig + (e & 1)
+      __syncthreads();   // P tiles and the row sums are complete
+#pragma unroll
+      for (int t = 0; t < QT; ++t)
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int j = t * 8 + 2 * tig + i;
+          lr[t][i] = lr[t][i] * al[t][i] + ((redl[j] + redl[16 + j]) + (redl[32 + j] + redl[48 + j]));
+        }
+      // ---- O^T = O^T * alpha + V^T P^T: A = V^T (16 dims x 16 keys, transposed loads of the V
+      // tile), B = P^T (16 keys x 8 query rows), for this warp's dimensions and every query tile
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
         for (int t = 0; t < QT; ++t)
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const int j = t * 8 + 2 * tig + (e & 1);
-            if (j < q && fits) {
-              const int dim = db + 16 * mt + g + 8 * (e >> 1);
-              p.part_o[((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + slot) * HD + dim] = O[mt][t][e] + Ol[mt][t][e];
-            }
+            O[mt][t][e] *= al[t][e & 1];
+            Ol[mt][t][e] *= al[t][e & 1];
           }
-      if (p.trace.rec) t_part = globaltimer_ns();
-      // the CTA's stores, then one release/acquire counter update by thread 0
-      __syncthreads();
-      if (tid == 0) *s_last = (atomic_add_acq_rel_gpu(p.counters + sl * H + h, 1) == nseg - 1);
-      __syncthreads();
-      if (*s_last && fits) {
-        // ---- merge the pair's partials: w[j][s] = exp(m_s - max m), L_j = sum_s w[j][s] l_s,
-        // O_j = (sum_s w[j][s] o_s) / L_j.  Each thread takes (row, 4 dimensions) pairs, two
-        // per round; a round's partial outputs are requested together with the statistics
-        // (first round), so the merge costs one round trip per round.
-        constexpr int PR = 2;                           // pairs per thread per round
-        const int npairs = q * D4;
-        for (int base = 0; base < npairs; base += 128 * PR) {
-          float4 v[PR][ATT_SEG_MAX];
+      if (ok) {
 #pragma unroll
-          for (int pp = 0; pp < PR; ++pp) {
-            const int t = base + tid + 128 * pp;
-            if (t < npairs) {
-              const int j = t / D4, d4 = t % D4;
-              const float4* po =
-                  reinterpret_cast<const float4*>(p.part_o + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair) * HD) + d4;
+        for (int kk = 0; kk < ATT_UNIT / 16; ++kk) {
+          uint32_t va[MT][4];
 #pragma unroll
-              for (int s2 = 0; s2 < ATT_SEG_MAX; ++s2)
-                if (s2 < nseg) v[pp][s2] = __ldcg(po + (size_t)s2 * D4);
-            }
-          }
-          if (base == 0) {
-            for (int t = tid; t < q * nseg; t += 128) {
-              const int j = t / nseg, s2 = t % nseg;
-              const float2 m2 = __ldcg(reinterpret_cast<const float2*>(
-                  p.part_ml + ((size_t)(sl * q + j) * H * ATT_SEG_MAX + pair + s2) * 2));
-              ms[j * ATT_SEG_MAX + s2] = m2.x;
-              ls[j * ATT_SEG_MAX + s2] = m2.y;
-            }
-            __syncthreads();
-            if (tid < q) {
-              float mx = -INFINITY;
-              for (int s2 = 0; s2 < nseg; ++s2) mx = fmaxf(mx, ms[tid * ATT_SEG_MAX + s2]);
-              float L = 0.f;
-              for (int s2 = 0; s2 < nseg; ++s2) {
-                const float m = ms[tid * ATT_SEG_MAX + s2];
-                const float w = (m == -INFINITY) ? 0.f : __expf(m - mx);
-                wg[tid * ATT_SEG_MAX + s2] = w;
-                L += w * ls[tid * ATT_SEG_MAX + s2];
-              }
-              inv[tid] = 1.0f / L;
-            }
-            __syncthreads();
+          for (int mt = 0; mt < MT; ++mt) {
+            const int key = kk * 16 + r8 + 8 * (mi >> 1);
+            const int dim = db + 16 * mt + 8 * (mi & 1);
+            const int hh = dim >> 6, cc = (dim & 63) >> 3;
+            ldsm_x4_t(smem_u32(Vt + hh * C::HALF_BYTES + key * 128 + ((cc ^ (key & 7)) << 4)), va[mt][0], va[mt][1],
+                      va[mt][2], va[mt][3]);
           }
 #pragma unroll
-          for (int pp = 0; pp < PR; ++pp) {
-            const int t = base + tid + 128 * pp;
-            if (t >= npairs) continue;
-            const int j = t / D4, d4 = t % D4;
-            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int t = 0; t < QT; ++t) {
+            uint32_t ph0, ph1, pl0, pl1;   // P rows t*8 .. t*8+7, keys kk*16 ..: hi (0, 1), lo (2, 3)
+            const uint8_t* psrc = (mi >> 1) ? Pl : Ph;
+            ldsm_x4(smem_u32(psrc + (t * 8 + r8) * C::PSTRIDE + (kk * 16 + 8 * (mi & 1)) * 2), ph0, ph1, pl0, pl1);
 #pragma unroll
-            for (int s2 = 0; s2 < ATT_SEG_MAX; ++s2) {
-              if (s2 < nseg) {
-                const float w = wg[j * ATT_SEG_MAX + s2];
-                a.x += w * v[pp][s2].x;
-                a.y += w * v[pp][s2].y;
-                a.z += w * v[pp][s2].z;
-                a.w += w * v[pp][s2].w;
-              }
+            for (int mt = 0; mt < MT; ++mt) {
+              mma_bf16_16816(O[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], ph0, ph1);
+              mma_bf16_16816(Ol[mt][t], va[mt][0], va[mt][1], va[mt][2], va[mt][3], pl0, pl1);
             }
-            const float iv = inv[j];
-            const float4 o = make_float4(a.x * iv, a.y * iv, a.z * iv, a.w * iv);
-            const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + 4 * d4;
-            *reinterpret_cast<float4*>(p.out + idx) = o;
-            const __nv_bfloat16 h0 = __float2bfloat16_rn(o.x), h1 = __float2bfloat16_rn(o.y);
-            const __nv_bfloat16 h2 = __float2bfloat16_rn(o.z), h3 = __float2bfloat16_rn(o.w);
-            uint2 hi, lo;
-            hi.x = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-            hi.y = (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
-            lo.x = pack_bf16(o.x - __bfloat162float(h0), o.y - __bfloat162float(h1));
-            lo.y = pack_bf16(o.z - __bfloat162float(h2), o.w - __bfloat162float(h3));
-            *reinterpret_cast<uint2*>(p.out_hi + idx) = hi;
-            *reinterpret_cast<uint2*>(p.out_lo + idx) = lo;
           }
         }
-        if (tid == 0) p.counters[sl * H + h] = 0;
-        ++merges;
-        if (p.trace.rec) t_merge = globaltimer_ns();
-        __syncthreads();   // merge scratch free again
       }
-      if (k + 1 < n) {     // the next unit starts the next pair
-        seg_first = u + 1;
-        locate(u + 1, sl, h, c);
+      __syncthreads();   // the stage, P and the row statistics are consumed
+      if (tid == 0 && isu.pi < npairs && !*abort_flag) {   // refill the freed stage, extend the L2 window
+        bool committed;
+        issue(issued, unit_row(isu, committed));
+        advance(isu);
+        ++issued;
+        if (pfc.pi < npairs) {
+          prefetch(unit_row(pfc, committed));
+          advance(pfc);
+        }
       }
-    } else {
-      ++c;
     }
+
+    // ---- this CTA's partial for the pair into its own shared memory (the Q and P tiles
+    // are free): O^T[mt][t][e] is dimension db + 16*mt + g + 8*(e >> 1) of query row
+    // t*8 + 2*tig + (e & 1); a CTA without units of the pair leaves (-inf, 0, 0)
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+      for (int t = 0; t < QT; ++t)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          po[(t * 8 + 2 * tig + (e & 1)) * HD + db + 16 * mt + g + 8 * (e >> 1)] = O[mt][t][e] + Ol[mt][t][e];
+    if (warp == 0 && g == 0) {
+#pragma unroll
+      for (int t = 0; t < QT; ++t)
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          pml[(t * 8 + 2 * tig + i) * 2] = mr[t][i];
+          pml[(t * 8 + 2 * tig + i) * 2 + 1] = lr[t][i];
+        }
+    }
+    if (p.trace.rec) t_part = globaltimer_ns();
+    cluster_sync_all();   // the cluster's cs partials of the pair are complete
+    // ---- merge this CTA's share of the pair's (row, 4 dimensions) outputs over the cs
+    // partials, read in rank order from the cluster's shared memory: w_r = exp(m_r - max m),
+    // L = sum_r w_r l_r, O = (sum_r w_r o_r) / L
+    {
+      const int items = q * D4, i0 = items * rank / CS, i1 = items * (rank + 1) / CS;
+      for (int it = i0 + tid; it < i1; it += 128) {
+        const int j = it / D4, d4 = it - j * D4;
+        const uint32_t a_ml = smem_u32(pml + 2 * j), a_o = smem_u32(po + j * HD + 4 * d4);
+        float2 ml[ATT_CS_MAX];
+        float4 ov[ATT_CS_MAX];
+#pragma unroll
+        for (int r = 0; r < ATT_CS_MAX; ++r)
+          if (r < CS) {
+            ml[r] = ld_dsmem_f2(mapa_shared(a_ml, r));
+            ov[r] = ld_dsmem_f4(mapa_shared(a_o, r));
+          }
+        float mx = -INFINITY;
+#pragma unroll
+        for (int r = 0; r < ATT_CS_MAX; ++r)
+          if (r < CS) mx = fmaxf(mx, ml[r].x);
+        float L = 0.f;
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int r = 0; r < ATT_CS_MAX; ++r)
+          if (r < CS) {
+            const float w = (ml[r].x == -INFINITY) ? 0.f : __expf(ml[r].x - mx);
+            L += w * ml[r].y;
+            a.x += w * ov[r].x;
+            a.y += w * ov[r].y;
+            a.z += w * ov[r].z;
+            a.w += w * ov[r].w;
+          }
+        const float iv = 1.0f / L;
+        const float4 o = make_float4(a.x * iv, a.y * iv, a.z * iv, a.w * iv);
+        const size_t idx = (size_t)(sl * q + j) * p.out_ld + h * HD + 4 * d4;
+        *reinterpret_cast<float4*>(p.out + idx) = o;
+        const __nv_bfloat16 h0 = __float2bfloat16_rn(o.x), h1 = __float2bfloat16_rn(o.y);
+        const __nv_bfloat16 h2 = __float2bfloat16_rn(o.z), h3 = __float2bfloat16_rn(o.w);
+        uint2 hi, lo;
+        hi.x = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+        hi.y = (uint32_t)__bfloat16_as_ushort(h2) | ((uint32_t)__bfloat16_as_ushort(h3) << 16);
+        lo.x = pack_bf16(o.x - __bfloat162float(h0), o.y - __bfloat162float(h1));
+        lo.y = pack_bf16(o.z - __bfloat162float(h2), o.w - __bfloat162float(h3));
+        *reinterpret_cast<uint2*>(p.out_hi + idx) = hi;
+        *reinterpret_cast<uint2*>(p.out_lo + idx) = lo;
+      }
+    }
+    if (p.trace.rec) t_merge = globaltimer_ns();
+    ++pairs_done;
+    cluster_sync_all();   // every CTA of the cluster has read this CTA's partial
   }
   if (*abort_flag && tid == 0) {   // let the copies in flight land before the CTA exits
     for (int i = max(0, issued - ATT_STAGES); i < issued; ++i) {
@@ -550,7 +518,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const __grid_constant__ 
     }
   }
   if (tid == 0 && p.trace.rec)
-    trace_write(p.trace, merges | ((unsigned)n << 8), t_entry, t_wait, t_k, t_part, t_merge, globaltimer_ns());
+    trace_write(p.trace, pairs_done | ((unsigned)k << 8), t_entry, t_wait, t_k, t_part, t_merge, globaltimer_ns());
 }
 
 // ---- prefill attention ----------------------------------------------------------------
@@ -773,34 +741,97 @@ __global__ void __launch_bounds__(128) prefill_attention_kernel(const __grid_con
   }
 }
 
-size_t attention_smem_bytes(int hd) { return hd == 64 ? AttCfg<64>::SMEM : AttCfg<128>::SMEM; }
+size_t attention_smem_bytes(int hd, int q) {
+  if (hd == 64) return q <= 8 ? AttCfg<64, 1>::SMEM : AttCfg<64, 2>::SMEM;
+  return q <= 8 ? AttCfg<128, 1>::SMEM : AttCfg<128, 2>::SMEM;
+}
+
+namespace {
+// most clusters of cs CTAs resident at once, per decode kernel instance (hd 64 / 128,
+// one or two query tiles) and cs = 1 .. ATT_CS_MAX; 0 = that cluster size cannot launch
+int g_att_clusters[2][2][ATT_CS_MAX + 1];
+bool g_att_clusters_known = false;
+int g_att_cs_cap = ATT_CS_MAX;   // SDSAT_ATT_CLUSTER_MAX: the largest cluster size launch_attention may pick
+
+template <int HD, int QT>
+cudaError_t prepare_decode_kernel(int (&maxc)[ATT_CS_MAX + 1]) {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(attention_kernel<HD, QT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)AttCfg<HD, QT>::SMEM)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(attention_kernel<HD, QT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
+      cudaSuccess)
+    return e;
+  for (int cs = 1; cs <= ATT_CS_MAX; ++cs) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cs * 64);
+    cfg.blockDim = dim3(128);
+    cfg.dynamicSmemBytes = AttCfg<HD, QT>::SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, attention_kernel<HD, QT>, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();   // this cluster size is not available: never chosen
+      n = 0;
+    }
+    maxc[cs] = n;
+  }
+  return cudaSuccess;
+}
+}  // namespace
 
 cudaError_t attention_prepare() {
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(attention_kernel<64, 1>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(attention_kernel<64, 2>, a, (int)AttCfg<64>::SMEM)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(attention_kernel<128, 1>, a, (int)AttCfg<128>::SMEM)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(attention_kernel<128, 2>, a, (int)AttCfg<128>::SMEM)) != cudaSuccess) return e;
+  if (!g_att_clusters_known) {
+    const char* cap = std::getenv("SDSAT_ATT_CLUSTER_MAX");
+    if (cap && cap[0]) g_att_cs_cap = std::max(1, std::min(ATT_CS_MAX, std::atoi(cap)));
+    if ((e = prepare_decode_kernel<64, 1>(g_att_clusters[0][0])) != cudaSuccess) return e;
+    if ((e = prepare_decode_kernel<64, 2>(g_att_clusters[0][1])) != cudaSuccess) return e;
+    if ((e = prepare_decode_kernel<128, 1>(g_att_clusters[1][0])) != cudaSuccess) return e;
+    if ((e = prepare_decode_kernel<128, 2>(g_att_clusters[1][1])) != cudaSuccess) return e;
+    g_att_clusters_known = true;
+  }
   if ((e = cudaFuncSetAttribute(prefill_attention_kernel<64>, a, (int)PfAttCfg<64>::SMEM)) != cudaSuccess) return e;
   return cudaFuncSetAttribute(prefill_attention_kernel<128>, a, (int)PfAttCfg<128>::SMEM);
 }
 
-cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl) {
-  // One wave of two CTAs per SM.  A pair of nu units is shared by at most
-  // (nu-1)P/U + 2 <= P/H + 2 CTAs, so P <= 14 H keeps that within ATT_SEG_MAX.
-  const long long units_max = (long long)p.nb * p.H * ((p.cap + ATT_UNIT - 1) / ATT_UNIT);
-  const int grid = (int)std::min<long long>(std::min(2 * num_sms, (ATT_SEG_MAX - 2) * p.H), units_max);
+cudaError_t launch_attention(const AttnParams& p0, int num_sms, cudaStream_t st, bool pdl) {
+  // One cluster per (sequence, head) pair, of the largest size cs that leaves room for
+  // ATT_SPARE_CLUSTERS more clusters among the CTAs resident at once: clusters are placed
+  // whole within one GPC, and grids that filled the GPU left some clusters waiting for
+  // a second wave.  If not even pairs of CTAs fit, single CTAs (as many as are resident
+  // at once) take several pairs each.
+  AttnParams p = p0;
+  const int pairs = p.nb * p.H;
+  const int(&maxc)[ATT_CS_MAX + 1] = g_att_clusters[p.hd == 128][p.q > 8];
+  const int resident = maxc[1] > 0 ? maxc[1] : 2 * num_sms;
+  p.cs = 1;
+  for (int cs = g_att_cs_cap; cs >= 2; --cs)
+    if (maxc[cs] >= pairs && cs * (pairs + ATT_SPARE_CLUSTERS) <= resident) {
+      p.cs = cs;
+      break;
+    }
+  p.nclusters = p.cs > 1 ? pairs : std::max(1, std::min(pairs, resident));
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(p.nclusters * p.cs);
   cfg.blockDim = dim3(128);
-  cfg.dynamicSmemBytes = attention_smem_bytes(p.hd);
+  cfg.dynamicSmemBytes = attention_smem_bytes(p.hd, p.q);
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = pdl ? 2 : 1;
   const bool one = p.q <= 8;
   if (p.hd == 64) return one ? cudaLaunchKernelEx(&cfg, attention_kernel<64, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<64, 2>, p);
   return one ? cudaLaunchKernelEx(&cfg, attention_kernel<128, 1>, p) : cudaLaunchKernelEx(&cfg, attention_kernel<128, 2>, p);

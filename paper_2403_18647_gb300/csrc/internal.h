@@ -108,7 +108,7 @@ cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl);
 // ---- attention -------------------------------------------------------------
 constexpr int ATT_UNIT = 64;          // keys per work unit: one TMA box of cache rows
 constexpr int ATT_MAX_CAP = 32768;    // KV capacity (slots per sequence) the kernel supports
-constexpr int ATT_SEG_MAX = 16;       // CTAs that may share one (sequence, head): partial slots per pair
+constexpr int ATT_CS_MAX = 16;        // CTAs of one cluster: the most that share one (sequence, head)
 #define SDSAT_ATT_MAXQ 16
 struct AttnParams {
   CUtensorMap kmap;     // the K cache as a 2-D tensor [rows][hd] bf16, boxes of 64 dims x ATT_UNIT rows
@@ -123,15 +123,14 @@ struct AttnParams {
   int out_ld;
   __nv_bfloat16* out_hi;    // the same as bf16 hi + lo (the O projection's operand)
   __nv_bfloat16* out_lo;
-  float* part_o;        // [rows][H][ATT_SEG_MAX][hd]: one unnormalised partial output per CTA sharing a pair
-  float* part_ml;       // [rows][H][ATT_SEG_MAX][2]: its running max and exp-sum
-  int* counters;        // [nb][H], zero between launches
+  int cs, nclusters;    // set by launch_attention: CTAs per cluster, clusters in the grid
   uint32_t* err;
   Trace trace;
 };
-size_t attention_smem_bytes(int hd);
-cudaError_t attention_prepare();   // set smem attributes (idempotent)
-// grid: min(2 * num_sms, 14 * H) CTAs, so at most ATT_SEG_MAX CTAs share one (sequence, head)
+size_t attention_smem_bytes(int hd, int q);
+cudaError_t attention_prepare();   // smem and cluster attributes, co-resident cluster counts (idempotent)
+// grid: nclusters clusters of cs CTAs, all resident at once; cluster c takes the
+// (sequence, head) pairs c, c + nclusters, ...; its CTAs split each pair's keys
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl);
 
 // Causal attention of M consecutive prompt positions of sequence seq (a prefill chunk at

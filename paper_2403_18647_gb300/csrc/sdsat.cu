@@ -123,9 +123,6 @@ struct sdsat_ctx {
   int* gemm_counters = nullptr;
   float* ssq = nullptr;        // [SDSAT_MAX_ROWS][ssq_ld] per-tile sums of h^2 (RMSNorm folded into the GEMMs)
   int ssq_ld = 0;
-  float* att_part_o = nullptr;
-  float* att_part_ml = nullptr;
-  int* att_counters = nullptr;
   int* acc_targets = nullptr;
   int* acc_counters = nullptr;
   int* tree_pos = nullptr;     // [SDSAT_MAX_ROWS] tree block positions (len + depth)
@@ -390,9 +387,6 @@ sdsat_status forward(sdsat_ctx* c, sdsat_kv* kv, int seq0, int nb, int q, const 
     a.out_ld = R;
     a.out_hi = c->x_hi[X_ATTN];
     a.out_lo = c->x_lo[X_ATTN];
-    a.part_o = c->att_part_o;
-    a.part_ml = c->att_part_ml;
-    a.counters = c->att_counters;
     a.err = c->err;
     a.trace = next_trace(c, K_ATTENTION);
     if (timed(c, K_ATTENTION, [&] { return launch_attention(a, c->num_sms, st, c->pdl); }) != cudaSuccess)
@@ -651,9 +645,7 @@ sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void*
             dalloc(c, &c->qbuf, (size_t)rows * R) && dalloc(c, &c->attn, (size_t)rows * R) &&
             dalloc(c, &c->act, (size_t)rows * F) && dalloc(c, &c->partials, (size_t)c->num_sms * 2 * 2 * 64 * 128) &&
             dalloc(c, &c->gemm_counters, MAX_GEMM_TILES) &&
-            dalloc(c, &c->att_part_o, (size_t)rows * cfg->n_heads * ATT_SEG_MAX * cfg->head_dim) &&
-            dalloc(c, &c->att_part_ml, (size_t)rows * cfg->n_heads * ATT_SEG_MAX * 2) &&
-            dalloc(c, &c->att_counters, (size_t)rows * cfg->n_heads) && dalloc(c, &c->acc_targets, rows) &&
+            dalloc(c, &c->acc_targets, rows) &&
             dalloc(c, &c->acc_counters, rows) && dalloc(c, &c->adaptive, SDSAT_MAX_ADAPTIVE) &&
             dalloc(c, &c->tree_pos, rows) && dalloc(c, &c->tree_anc, rows) &&
             dalloc(c, &c->tree_ws, (size_t)rows * TREE_WS_STRIDE) &&
@@ -1099,11 +1091,6 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   if (b < 1 || q < 1 || q > SDSAT_MAX_Q || b * q > SDSAT_MAX_ROWS || (hd != 64 && hd != 128) || H < 1 || cap < 1 ||
       cap > ATT_MAX_CAP)
     return SDSAT_EINVAL;
-  // the partial-result workspace was sized at create for SDSAT_MAX_ROWS rows of the model's heads
-  const size_t have = (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * ATT_SEG_MAX;
-  if ((size_t)b * q * H * ATT_SEG_MAX * hd > have * c->cfg.head_dim || (size_t)b * q * H * ATT_SEG_MAX > have ||
-      (size_t)b * H > (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads)
-    return SDSAT_EINVAL;
   AttnParams a;
   std::memset(&a, 0, sizeof(a));
   if (!aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) || (long long)b * H * cap > 0x7FFFFFFFll)
@@ -1125,9 +1112,6 @@ sdsat_status sdsat_op_attention(sdsat_ctx* c, const float* q_dev, const void* k_
   if ((size_t)b * q * H * hd > (size_t)SDSAT_MAX_ROWS * c->cfg.n_heads * c->cfg.head_dim) return SDSAT_EINVAL;
   a.out_hi = c->x_hi[X_ATTN];
   a.out_lo = c->x_lo[X_ATTN];
-  a.part_o = c->att_part_o;
-  a.part_ml = c->att_part_ml;
-  a.counters = c->att_counters;
   a.err = c->err;
   return timed(c, K_ATTENTION_OP, [&] { return launch_attention(a, c->num_sms, c->stream, c->pdl); }) == cudaSuccess
              ? SDSAT_OK
