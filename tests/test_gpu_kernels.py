@@ -110,6 +110,11 @@ ATT_CASES = [
     (1, 1, 4, 64, [0], 64), (1, 6, 4, 64, [5], 64), (1, 6, 4, 64, [122], 256), (1, 6, 4, 64, [123], 256),
     (1, 16, 2, 128, [300], 512), (3, 6, 4, 128, [0, 127, 250], 300), (2, 11, 4, 64, [129, 1000], 1100),
     (4, 6, 32, 128, [1024, 1100, 1200, 1270], 1290),
+    # more (sequence, head) pairs than fit as clusters: single CTAs, some taking two pairs
+    # (q <= 8: 512 pairs; q = 9: 448 pairs), or one pair each (256 pairs)
+    (16, 4, 32, 128, [0, 1, 63, 64, 65, 100, 127, 128, 200, 257, 300, 383, 450, 511, 600, 630], 640),
+    (7, 9, 64, 64, [0, 5, 64, 130, 200, 255, 310], 320),
+    (8, 8, 32, 128, [700, 10, 333, 64, 512, 1, 600, 129], 710),
 ]
 
 
