@@ -24,7 +24,9 @@ pipelined the pipelined variant (not a step of the paper): the verification
 Pins (tests/test_oracle_*.py) tie every function to something other than
 itself: closed forms, invariants the method fixes (greedy SDSAT output equals
 plain greedy output, Sec. 2.1.1; a q-row block equals q sequential steps),
-brute force on tiny inputs and published known-answer vectors.  The
-end-to-end logits of a randomly initialised model have no printed values
-anywhere: beyond those invariants they are "parity unpinned".
+brute force on tiny inputs and published known-answer vectors; the decoder
+forward's composition is pinned on weight settings where it reduces to library
+routines (zeroed branches, a single key, one causal attention layer).  The
+end-to-end logits of a randomly initialised model with every branch on have no
+printed values anywhere: beyond those pins they are "parity unpinned".
 """
