@@ -60,9 +60,9 @@ struct AttCfg {
   static constexpr int RED = 17;                         // floats per row of the row-reduction scratch
   // Q hi + lo tiles; once the CTA's units of a pair are done, its partial output [ROWS][HD] fp32
   static constexpr size_t OFF_Q = (size_t)ATT_STAGES * STAGE;
-  // P hi + lo tiles; once the units are done, the partial's row max and exp-sum [ROWS][2]
+  // P hi + lo tiles
   static constexpr size_t OFF_P = OFF_Q + 2 * ROWS * QSTRIDE;
-  static constexpr size_t OFF_RED = OFF_P + 2 * ROWS * PSTRIDE;                     // [16][RED]
+  static constexpr size_t OFF_RED = OFF_P + 2 * ROWS * PSTRIDE;   // [16][RED]: unit row max, sums; partial stats
   static constexpr size_t OFF_SEQ = OFF_RED + 16 * RED * 4;                         // len, units [64]
   static constexpr size_t OFF_ANC = OFF_SEQ + (64 + 64) * 4;                        // [16] visible block rows per row
   static constexpr size_t OFF_BAR = (OFF_ANC + 16 * 4 + 7) / 8 * 8;
@@ -109,8 +109,8 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
   float* po = reinterpret_cast<float*>(smem + C::OFF_Q);        // [ROWS][HD] partial output (after the units)
   uint8_t* Ph = smem + C::OFF_P;                    // bf16 [ROWS][ATT_UNIT] softmax numerators, hi part
   uint8_t* Pl = Ph + C::ROWS * C::PSTRIDE;
-  float* pml = reinterpret_cast<float*>(smem + C::OFF_P);       // [ROWS][2] partial row max, exp-sum (after the units)
-  float* red = reinterpret_cast<float*>(smem + C::OFF_RED);     // row-reduction scratch
+  float* red = reinterpret_cast<float*>(smem + C::OFF_RED);     // row-reduction scratch [4][16] max, [4][16] sums
+  float* pml = red + 128;                                       // [ROWS][2] partial row max, exp-sum (after the units)
   int* len_seq = reinterpret_cast<int*>(smem + C::OFF_SEQ);     // [64] committed length of each sequence
   int* nu_seq = len_seq + 64;                                   // [64] units per head of each sequence
   uint32_t* anc_s = reinterpret_cast<uint32_t*>(smem + C::OFF_ANC);   // [16] block rows row j sees (bit i)
@@ -318,14 +318,18 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
       // St[t][e] is the score of key kb + g + 8*(e >> 1) for query row t*8 + 2*tig + (e & 1).
       // mask: row j sees key slot kp iff kp < len, or kp = len + i for a block row i that
       // anc_s[j] marks (and kp < nkeys, j < q)
+      // (a unit of committed slots only is seen whole by every row; rows j >= q are never
+      // merged, so their unmasked scores of zero do no harm)
+      if (!ok || c0 + ATT_UNIT > len) {
 #pragma unroll
-      for (int t = 0; t < QT; ++t)
+        for (int t = 0; t < QT; ++t)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int j = t * 8 + 2 * tig + (e & 1);
-          const int kp = c0 + kb + g + 8 * (e >> 1);
-          if (!ok || j >= q || kp >= nkeys || (kp >= len && !((anc_s[j] >> (kp - len)) & 1u))) St[t][e] = -INFINITY;
-        }
+          for (int e = 0; e < 4; ++e) {
+            const int j = t * 8 + 2 * tig + (e & 1);
+            const int kp = c0 + kb + g + 8 * (e >> 1);
+            if (!ok || j >= q || kp >= nkeys || (kp >= len && !((anc_s[j] >> (kp - len)) & 1u))) St[t][e] = -INFINITY;
+          }
+      }
       // ---- the unit's row maxima: over the warp's lanes holding other keys (g), then the four
       // warps through shared memory; the running statistics stay in registers
       float* redm = red;          // [4 warps][16 rows] unit row maxima
@@ -345,7 +349,18 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
           redm[warp * 16 + t * 8 + 2 * tig + 1] = mx[t][1];
         }
       }
-      __syncthreads();
+      __syncthreads();   // every warp is also done with the previous unit (its stage, P, red)
+      if (tid == 0 && k >= 1 && isu.pi < npairs && !*abort_flag) {
+        // refill the previous unit's stage with unit k + 1, extend the L2 window
+        bool committed;
+        issue(issued, unit_row(isu, committed));
+        advance(isu);
+        ++issued;
+        if (pfc.pi < npairs) {
+          prefetch(unit_row(pfc, committed));
+          advance(pfc);
+        }
+      }
       float al[QT][2];   // rescale of what the units before contributed
 #pragma unroll
       for (int t = 0; t < QT; ++t)
@@ -425,21 +440,11 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
           }
         }
       }
-      __syncthreads();   // the stage, P and the row statistics are consumed
-      if (tid == 0 && isu.pi < npairs && !*abort_flag) {   // refill the freed stage, extend the L2 window
-        bool committed;
-        issue(issued, unit_row(isu, committed));
-        advance(isu);
-        ++issued;
-        if (pfc.pi < npairs) {
-          prefetch(unit_row(pfc, committed));
-          advance(pfc);
-        }
-      }
     }
 
-    // ---- this CTA's partial for the pair into its own shared memory (the Q and P tiles
-    // are free): O^T[mt][t][e] is dimension db + 16*mt + g + 8*(e >> 1) of query row
+    // ---- this CTA's partial for the pair into its own shared memory (the output over the
+    // Q tiles, which no warp reads any more; the statistics beside the row-reduction
+    // scratch): O^T[mt][t][e] is dimension db + 16*mt + g + 8*(e >> 1) of query row
     // t*8 + 2*tig + (e & 1); a CTA without units of the pair leaves (-inf, 0, 0)
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt)
