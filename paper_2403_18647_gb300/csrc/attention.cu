@@ -125,6 +125,10 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
   const int rank = (int)cluster_ctarank(), cl = (int)blockIdx.x / CS;
   const unsigned long long t_entry = p.trace.rec ? globaltimer_ns() : 0;
   pdl_trigger();
+  if (tid == 64) {   // the tensor maps into the TMA unit while the lengths are read
+    tma_prefetch_desc(&p.kmap);
+    tma_prefetch_desc(&p.vmap);
+  }
 
   // The committed lengths are final before this kernel can start: the block forward's
   // first kernel (RMSNorm) lets its dependents launch only after every earlier kernel
@@ -198,8 +202,6 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
   int issued = 0;
   Cursor isu{npairs, 0, 0}, pfc{npairs, 0, 0};
   if (tid == 0) {
-    tma_prefetch_desc(&p.kmap);
-    tma_prefetch_desc(&p.vmap);
     pol = l2_policy_evict_first();
     // Tiles of committed slots do not depend on the QKV projection: the first ones go
     // to the ring now, the next ATT_PREFETCH into L2 (and one more each time the ring is

@@ -283,6 +283,12 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   unsigned long long t_wait = 0;
   const long long g0 = (long long)cta * T / p.P, g1 = (long long)(cta + 1) * T / p.P;
 
+  if (threadIdx.x == 64) {   // the tensor maps into the TMA unit while the CTA sets up
+    const int nmaps = p.map_mode == MAP_QKV3 ? 3 : (p.map_mode == MAP_GATEUP ? 2 : 1);
+    for (int i = 0; i < nmaps; ++i) tma_prefetch_desc(&p.tmap[i]);
+    tma_prefetch_desc(&p.tmap_x[0]);
+    tma_prefetch_desc(&p.tmap_x[1]);
+  }
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
@@ -308,10 +314,6 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   if (warp == 0) {
     // ------------------------------------------------ weight + activation stream (TMA)
     if (lane == 0) {
-      const int nmaps = p.map_mode == MAP_QKV3 ? 3 : (p.map_mode == MAP_GATEUP ? 2 : 1);
-      for (int i = 0; i < nmaps; ++i) tma_prefetch_desc(&p.tmap[i]);
-      tma_prefetch_desc(&p.tmap_x[0]);
-      tma_prefetch_desc(&p.tmap_x[1]);
       const uint64_t pol_w = l2_policy_evict_first();   // weights: read once per step
       const uint64_t pol_x = l2_policy_evict_last();    // activations: read by every CTA
       constexpr uint32_t TX = C::W_BYTES + 2 * C::X_BYTES;
