@@ -61,8 +61,8 @@ WORKLOADS = {
 # DRAM bytes (read + write) per algorithmic byte of the skinny GEMM, from one ncu capture
 # (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.35 MB of traffic for
 # 181.0 MB of weights + operand + output.  Applied to the average launch of the step.
-GEMM_TRAFFIC_RATIO = 186.33 / 181.0
-GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.33 MB for 181.0 MB "
+GEMM_TRAFFIC_RATIO = 186.57 / 181.0
+GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.57 MB for 181.0 MB "
                        "algorithmic, profiles/gemm_gateup_4096x22016_m6.md), ratio scaled to the average launch; "
                        "bytes per launch")
 
