@@ -113,7 +113,12 @@ typedef struct {
 /* Validate `cfg`, record the weight pointers, build the TMA descriptors and the
  * RoPE table, allocate the library-owned workspaces.  `stream` is a cudaStream_t
  * (NULL = legacy default stream).  Synchronous.  Errors: EINVAL (bad config or
- * pointer), EUNSUPPORTED (head_dim, GQA), ENOMEM, ECUDA. */
+ * pointer), EUNSUPPORTED (head_dim, GQA), ENOMEM, ECUDA.
+ * Environment: SDSAT_NO_PDL=1 (read at each create) launches this context's kernels
+ * without programmatic dependent launch, for tools that cannot follow it;
+ * SDSAT_ATT_CLUSTER_MAX=n (read at the first create of the process) caps the
+ * attention's thread-block cluster size at n in 1..16 for tuning sweeps (default
+ * 16; the size itself is chosen per launch). */
 SDSAT_API sdsat_status sdsat_create(const sdsat_config* cfg, const sdsat_weights* w, void* stream,
                           sdsat_ctx** out);
 SDSAT_API void sdsat_destroy(sdsat_ctx* ctx);
