@@ -434,8 +434,9 @@ SDSAT_API sdsat_status sdsat_profile_end(sdsat_ctx* ctx, sdsat_kernel_stat* out,
  *   [4], [5], [6] kernel-specific marks (0 = not reached), [7] at exit.
  * GEMM: marks = first MMA issued, accumulator of the CTA's last tile ready, that tile
  * reduced (or handed to another CTA); flags = 1 if this CTA reduced it | contributors << 8.
- * Attention: marks = K tile landed, partial result written, merge weights ready (merging
- * CTA only); flags = 1 for the merging CTA | number of chunks << 8.
+ * Attention: marks = first K/V tile usable, the CTA's partial of its last (sequence, head)
+ * pair written, that pair's share of the merged output stored; flags = pairs taken |
+ * units of 64 slots << 8.
  * begin allocates room for max_records records (call it outside any graph capture); end
  * synchronises, copies up to max_records records to host memory and frees the buffer. */
 #define SDSAT_TRACE_WORDS 8
