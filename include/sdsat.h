@@ -374,6 +374,17 @@ SDSAT_API sdsat_status sdsat_op_attention(sdsat_ctx* ctx, const float* q_dev, co
  * layer.  For tests that check a forward stage by stage.  Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_debug_workspace(sdsat_ctx* ctx, int which, int rows, float* dst_dev);
 
+/* The attention grid sdsat_block_forward and sdsat_op_attention launch for `pairs`
+ * (sequence, head) pairs (host only, no GPU): one thread-block cluster of *cs CTAs per
+ * pair, *nclusters = pairs, for the largest cs <= min(cs_cap, 16) with
+ * max_clusters[cs] >= pairs and cs * (pairs + 8) <= max_clusters[1] (the CTAs resident
+ * at once, else 2 * num_sms); otherwise *cs = 1 and *nclusters = min(pairs, resident),
+ * each CTA taking several pairs.  max_clusters[c] (c = 1..16, host array of 17 entries,
+ * [0] unused) = the most clusters of c CTAs the device holds at once, as
+ * cudaOccupancyMaxActiveClusters reports it for the attention kernel.  Errors: EINVAL. */
+SDSAT_API sdsat_status sdsat_attention_grid(int pairs, const int32_t* max_clusters, int cs_cap, int num_sms,
+                                            int* cs, int* nclusters);
+
 /* Test hook for failure detection: one kernel waits on a barrier that nothing
  * completes, through the bounded wait every kernel of the library uses.  After its
  * limit (2 s) it sets device bit TIMEOUT and returns; nothing faults and the

@@ -100,6 +100,7 @@ def _lib():
             "sdsat_op_exp": [P, P, P, I],
             "sdsat_debug_workspace": [P, I, I, P],
             "sdsat_debug_wait_timeout": [P],
+            "sdsat_attention_grid": [I, P, I, I, ctypes.POINTER(I), ctypes.POINTER(I)],
         }
         for name, args in sig.items():
             fn = getattr(lib, name)
@@ -137,6 +138,16 @@ def _ptr(t) -> Optional[int]:
 def _check(status: int, what: str):
     if status != 0:
         raise SdsatError(status, what)
+
+
+def attention_grid(pairs: int, max_clusters, cs_cap: int = 16, num_sms: int = 152):
+    """(cluster size, clusters) the attention launches for `pairs` (sequence, head) pairs,
+    given max_clusters[c] = the most clusters of c CTAs resident at once (c = 1..16)."""
+    arr = (ctypes.c_int32 * 17)(0, *[int(v) for v in list(max_clusters)[1:17]])
+    cs, nc = ctypes.c_int(0), ctypes.c_int(0)
+    _check(_lib().sdsat_attention_grid(pairs, ctypes.cast(arr, ctypes.c_void_p), cs_cap, num_sms,
+                                       ctypes.byref(cs), ctypes.byref(nc)), "sdsat_attention_grid")
+    return cs.value, nc.value
 
 
 def _stream():

@@ -808,23 +808,25 @@ cudaError_t attention_prepare() {
   return cudaFuncSetAttribute(prefill_attention_kernel<128>, a, (int)PfAttCfg<128>::SMEM);
 }
 
-cudaError_t launch_attention(const AttnParams& p0, int num_sms, cudaStream_t st, bool pdl) {
+void attention_grid(int pairs, const int* maxc, int cs_cap, int num_sms, int* cs, int* nclusters) {
   // One cluster per (sequence, head) pair, of the largest size cs that leaves room for
   // ATT_SPARE_CLUSTERS more clusters among the CTAs resident at once: clusters are placed
   // whole within one GPC, and grids that filled the GPU left some clusters waiting for
   // a second wave.  If not even pairs of CTAs fit, single CTAs (as many as are resident
   // at once) take several pairs each.
-  AttnParams p = p0;
-  const int pairs = p.nb * p.H;
-  const int(&maxc)[ATT_CS_MAX + 1] = g_att_clusters[p.hd == 128][p.q > 8];
   const int resident = maxc[1] > 0 ? maxc[1] : 2 * num_sms;
-  p.cs = 1;
-  for (int cs = g_att_cs_cap; cs >= 2; --cs)
-    if (maxc[cs] >= pairs && cs * (pairs + ATT_SPARE_CLUSTERS) <= resident) {
-      p.cs = cs;
+  *cs = 1;
+  for (int c = std::min(cs_cap, ATT_CS_MAX); c >= 2; --c)
+    if (maxc[c] >= pairs && c * (pairs + ATT_SPARE_CLUSTERS) <= resident) {
+      *cs = c;
       break;
     }
-  p.nclusters = p.cs > 1 ? pairs : std::max(1, std::min(pairs, resident));
+  *nclusters = *cs > 1 ? pairs : std::max(1, std::min(pairs, resident));
+}
+
+cudaError_t launch_attention(const AttnParams& p0, int num_sms, cudaStream_t st, bool pdl) {
+  AttnParams p = p0;
+  attention_grid(p.nb * p.H, g_att_clusters[p.hd == 128][p.q > 8], g_att_cs_cap, num_sms, &p.cs, &p.nclusters);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.nclusters * p.cs);
   cfg.blockDim = dim3(128);

@@ -132,6 +132,9 @@ cudaError_t attention_prepare();   // smem and cluster attributes, co-resident c
 // grid: nclusters clusters of cs CTAs, all resident at once; cluster c takes the
 // (sequence, head) pairs c, c + nclusters, ...; its CTAs split each pair's keys
 cudaError_t launch_attention(const AttnParams& p, int num_sms, cudaStream_t st, bool pdl);
+// the grid launch_attention picks for `pairs` (sequence, head) pairs: maxc[c] = most
+// clusters of c CTAs resident at once (c = 1..ATT_CS_MAX), cluster size at most cs_cap
+void attention_grid(int pairs, const int* maxc, int cs_cap, int num_sms, int* cs, int* nclusters);
 
 // Causal attention of M consecutive prompt positions of sequence seq (a prefill chunk at
 // slots len[seq] .. len[seq]+M-1, already in the cache) over the cache: position i sees

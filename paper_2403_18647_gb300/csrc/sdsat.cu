@@ -1029,6 +1029,13 @@ sdsat_status sdsat_build_pipelined_block(sdsat_ctx* c, sdsat_kv* kv, const int32
              : SDSAT_ECUDA;
 }
 
+sdsat_status sdsat_attention_grid(int pairs, const int32_t* max_clusters, int cs_cap, int num_sms,
+                                  int* cs, int* nclusters) {
+  if (pairs < 1 || !max_clusters || cs_cap < 1 || num_sms < 1 || !cs || !nclusters) return SDSAT_EINVAL;
+  attention_grid(pairs, max_clusters, cs_cap, num_sms, cs, nclusters);
+  return SDSAT_OK;
+}
+
 sdsat_status sdsat_debug_wait_timeout(sdsat_ctx* c) {
   if (!c) return SDSAT_EINVAL;
   return launch_wait_timeout(c->err, c->stream) == cudaSuccess ? SDSAT_OK : SDSAT_ECUDA;
