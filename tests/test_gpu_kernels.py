@@ -233,7 +233,7 @@ def test_accept_nan_rows(accept_env):
 @pytest.mark.parametrize("T,top_p,top_k", [(0.2, 0.95, 0), (1.0, 0.95, 0), (1.0, 0.95, 10), (0.7, 0.5, 0),
                                            (1.0, 1.0, 0), (2.0, 0.0, 0), (0.2, 0.95, 1)])
 def test_accept_nucleus_bit_exact(accept_env, T, top_p, top_k):
-    """The acceptance kernel is bit-exact on identical logits (spec requirement)."""
+    """The acceptance kernel is bit-exact on identical logits (the required tolerance for it)."""
     V = accept_env.shape.vocab
     b, q = 2, 6
     for trial in range(3):
