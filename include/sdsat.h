@@ -53,7 +53,7 @@ typedef enum {
   SDSAT_ECAPACITY = 3,     /* batch, q, position or KV capacity limit exceeded */
   SDSAT_ECUDA = 4,         /* a CUDA runtime or driver call failed */
   SDSAT_EDEVICE = 5,       /* device-detected error bits were set (sdsat_get_error) */
-  SDSAT_EUNSUPPORTED = 6   /* a configuration this build does not implement */
+  SDSAT_EUNSUPPORTED = 6   /* a configuration this library does not implement */
 } sdsat_status;
 
 /* device error bits reported by sdsat_get_error */
@@ -76,7 +76,7 @@ typedef struct {
   int32_t n_layers;
   int32_t d_model;
   int32_t n_heads;
-  int32_t n_kv_heads;      /* must equal n_heads in this build (no grouped-query attention) */
+  int32_t n_kv_heads;      /* must equal n_heads (this library has no grouped-query attention) */
   int32_t head_dim;        /* 64 or 128 */
   int32_t ffn_dim;         /* SwiGLU hidden size */
   int32_t vocab;           /* including the semantic adaptive tokens (Sec. 3.2: ordinary ids) */
