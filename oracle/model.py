@@ -30,6 +30,11 @@ Readings where the paper is silent (all configurable):
     to q single-token steps, the invariant the method relies on).
 
 All arithmetic is fp64; weights are the bf16 values widened exactly.
+
+Diagnostic mode (KVCache(kv_bf16=True)): the K and V rows are rounded to bf16
+(round to nearest even) when written, as a cache stored in bf16 holds them; every
+other step stays fp64.  Comparing a bf16-cache implementation with this mode
+separates its arithmetic errors from the cache's storage precision.
 """
 from __future__ import annotations
 
@@ -143,15 +148,22 @@ class Weights:
         return a
 
 
-class KVCache:
-    """Per-layer K and V (fp64) for b sequences: [L][b][H][max_len][hd], plus len[b]."""
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """x rounded to the nearest bf16 value (ties to even), returned in fp64."""
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float64)).to(torch.bfloat16).to(torch.float64).numpy()
 
-    def __init__(self, shape, batch: int, max_len: int):
+
+class KVCache:
+    """Per-layer K and V (fp64) for b sequences: [L][b][H][max_len][hd], plus len[b].
+    kv_bf16: store the rows rounded to bf16 (the diagnostic mode of the module docstring)."""
+
+    def __init__(self, shape, batch: int, max_len: int, kv_bf16: bool = False):
         L, H, hd = shape.n_layers, shape.n_heads, shape.head_dim
         self.K = [np.zeros((batch, H, max_len, hd)) for _ in range(L)]
         self.V = [np.zeros((batch, H, max_len, hd)) for _ in range(L)]
         self.len = [0] * batch
         self.max_len = max_len
+        self.kv_bf16 = kv_bf16
 
     def copy(self) -> "KVCache":
         c = KVCache.__new__(KVCache)
@@ -159,6 +171,7 @@ class KVCache:
         c.V = [v.copy() for v in self.V]
         c.len = list(self.len)
         c.max_len = self.max_len
+        c.kv_bf16 = self.kv_bf16
         return c
 
 
@@ -193,6 +206,8 @@ def block_forward(W: Weights, kv: KVCache, seq: int, tokens: Sequence[int],
         v = linear(x, W.get("wv", l)).reshape(n, H, hd)
         q = rope(q, pos, shape.rope_theta)
         k = rope(k, pos, shape.rope_theta)
+        if kv.kv_bf16:
+            k, v = round_bf16(k), round_bf16(v)
         kv.K[l][seq][:, L0:L0 + n] = k.transpose(1, 0, 2)
         kv.V[l][seq][:, L0:L0 + n] = v.transpose(1, 0, 2)
         if visible is None:

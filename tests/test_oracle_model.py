@@ -157,3 +157,37 @@ def test_norm_gain_matters(tiny_shape, tiny_model_cpu, tiny_model_cpu_unit_gain)
     a = M.block_forward(_weights(tiny_shape, tiny_model_cpu), M.KVCache(tiny_shape, 1, 8), 0, [3])
     b = M.block_forward(_weights(tiny_shape, tiny_model_cpu_unit_gain), M.KVCache(tiny_shape, 1, 8), 0, [3])
     assert np.abs(a - b).max() > 1e-3
+
+
+def test_round_bf16_ties_to_even():
+    """bf16 keeps 8 significant bits: the spacing just above 1 is 2^-7."""
+    x = np.array([1.0, 1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, 1 + 2.0 ** -8 + 2.0 ** -20, -(1 + 2.0 ** -8),
+                  3.0 * 2.0 ** -130, 1.0 + 2.0 ** -7])
+    want = np.array([1.0, 1.0, 1 + 2.0 ** -6, 1 + 2.0 ** -7, -1.0, 3.0 * 2.0 ** -130, 1.0 + 2.0 ** -7])
+    np.testing.assert_array_equal(M.round_bf16(x), want)
+
+
+def test_bf16_cache_mode(tiny_shape, tiny_model_cpu):
+    """Diagnostic mode: cached K / V rows are bf16 values, a block still equals the
+    sequential steps bit for bit, and the logits move by the cache's rounding only."""
+    W = _weights(tiny_shape, tiny_model_cpu)
+    prompt = synth.prompt_ids(0, 5, 30, 4096).tolist()
+    blk = [7, 4096, 11, 2000, 4096, 8]
+    exact, rounded = M.KVCache(tiny_shape, 1, 64), M.KVCache(tiny_shape, 1, 64, kv_bf16=True)
+    M.prefill(W, exact, 0, prompt)
+    M.prefill(W, rounded, 0, prompt)
+    assert rounded.copy().kv_bf16
+    kv_a = rounded.copy()
+    la = M.block_forward(W, kv_a, 0, blk)
+    for l in range(tiny_shape.n_layers):
+        K = kv_a.K[l][0][:, :36]
+        np.testing.assert_array_equal(M.round_bf16(K), K)
+        assert not np.array_equal(M.round_bf16(exact.K[l][0][:, :30]), exact.K[l][0][:, :30])
+    kv_b = rounded.copy()
+    for j, t in enumerate(blk):
+        lj = M.block_forward(W, kv_b, 0, [t])
+        kv_b.len[0] += 1
+        np.testing.assert_array_equal(lj[0], la[j])
+    le = M.block_forward(W, exact.copy(), 0, blk)
+    d = np.abs(la - le).max()
+    assert 0 < d < 0.05 * np.abs(le).max(), d
