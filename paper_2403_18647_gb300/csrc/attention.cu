@@ -285,8 +285,9 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
       const int c0 = c * ATT_UNIT;                  // slot of the unit's first key
       const uint8_t* Kt = smem + (size_t)(k % ATT_STAGES) * C::STAGE;
       const uint8_t* Vt = Kt + C::TILE;
-      const bool ok = mbar_wait_bounded(&full[k % ATT_STAGES], (k / ATT_STAGES) & 1, abort_flag, p.err);
-      __syncwarp();   // lanes leave the polling loop at different times: reconverge
+      // one decision per warp (mma.sync needs every lane; a wait can run out for some only)
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[k % ATT_STAGES], (k / ATT_STAGES) & 1,
+                                                              abort_flag, p.err));
       if (k == 0 && p.trace.rec) t_k = globaltimer_ns();
 
       // ---- S^T = K Q^T for this warp's 16 keys: m16n8k16 with A = K (16 keys x 16 dims) and
@@ -619,8 +620,8 @@ __global__ void __launch_bounds__(128) prefill_attention_kernel(const __grid_con
   for (int u = 0; u < nu; ++u) {
     const uint8_t* Kt = smem + (size_t)(u % ATT_STAGES) * C::STAGE;
     const uint8_t* Vt = Kt + C::TILE;
-    const bool ok = mbar_wait_bounded(&full[u % ATT_STAGES], (u / ATT_STAGES) & 1, abort_flag, p.err);
-    __syncwarp();
+    const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(&full[u % ATT_STAGES], (u / ATT_STAGES) & 1,
+                                                            abort_flag, p.err));
     float s[8][4];
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;

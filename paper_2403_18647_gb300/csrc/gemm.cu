@@ -447,8 +447,9 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
         if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
       }
-      const bool got = mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err);
-      __syncwarp();   // lanes leave the polling loop at different times: reconverge
+      // the four epilogue warps decide together (lanes leave the polling loop at different
+      // times, and a wait can run out for some of them only)
+      const bool got = named_bar_and(1, 128, mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err));
       if (!got) break;
       tc_fence_after();
       const bool last_seg = g >= g1;
@@ -510,8 +511,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
               bulk_load_g2s(stages + (size_t)r * pbytes,
                             p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128, pbytes, red_bar);
             }
-            ok = mbar_wait_bounded(red_bar, ph, abort_flag, p.err);
-            __syncwarp();
+            ok = named_bar_and(1, 128, mbar_wait_bounded(red_bar, ph, abort_flag, p.err));
             ph ^= 1u;
             if (ok) {
               for (int u = 0; u < cnt; ++u) {

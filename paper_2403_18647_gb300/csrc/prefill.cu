@@ -167,8 +167,7 @@ __global__ void __launch_bounds__(192, 1) prefill_gemm_kernel(const __grid_const
     for (int t = blockIdx.x; t < T; t += P, ++seg) {
       const int wt = t / p.n_tblocks, tb = t % p.n_tblocks;
       const int buf = seg & 1;
-      const bool got = mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err);
-      __syncwarp();
+      const bool got = named_bar_and(1, 128, mbar_wait_bounded(&acc_full[buf], (seg >> 1) & 1, abort_flag, p.err));
       if (!got) break;
       tc_fence_after();
       const uint32_t lane_addr = tmem + ((uint32_t)(e * 32) << 16) + buf * PF_ACC;
