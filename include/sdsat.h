@@ -111,8 +111,11 @@ typedef struct {
 /* ---- lifetime ----------------------------------------------------------------- */
 
 /* Validate `cfg`, record the weight pointers, build the TMA descriptors and the
- * RoPE table, allocate the library-owned workspaces.  `stream` is a cudaStream_t
- * (NULL = legacy default stream).  Synchronous.  Errors: EINVAL (bad config or
+ * RoPE table, allocate the library-owned workspaces.  The model is the unmodified
+ * decoder the method runs (Abstract, Sec. 1: no structural change; Sec. 3.2: the
+ * adaptive tokens are ordinary vocabulary ids), so the configuration is a plain
+ * Llama configuration plus the adaptive ids; the paper prescribes no interface for
+ * it.  `stream` is a cudaStream_t (NULL = legacy default stream).  Synchronous.  Errors: EINVAL (bad config or
  * pointer), EUNSUPPORTED (head_dim, GQA), ENOMEM, ECUDA.
  * Environment: SDSAT_NO_PDL=1 (read at each create) launches this context's kernels
  * without programmatic dependent launch, for tools that cannot follow it;
@@ -126,7 +129,9 @@ SDSAT_API void sdsat_destroy(sdsat_ctx* ctx);
 /* Stream for all later compute calls on ctx (a cudaStream_t). */
 SDSAT_API sdsat_status sdsat_set_stream(sdsat_ctx* ctx, void* stream);
 
-/* Library-owned KV cache for `batch` sequences of up to `max_len` slots:
+/* Library-owned KV cache for `batch` sequences of up to `max_len` slots (the cache
+ * that Eq. 1 and Eq. 2 extend by q positions per pass and that Sec. 2.1.1's
+ * verification truncates to the accepted prefix; the paper states no layout):
  * K and V bf16 [n_layers][batch][n_heads][max_len][head_dim], and the committed
  * length len[batch] (int32, device, starts at 0).  Synchronous.
  * Errors: EINVAL, ENOMEM, ECAPACITY (max_len > max_position or > 32768). */
@@ -187,7 +192,8 @@ SDSAT_API sdsat_status sdsat_accept_greedy(sdsat_ctx* ctx, sdsat_kv* kv, const f
  * that any two implementations agree bit for bit:
  *   s_i = (l_i - max l) / temperature (fp32), w_i = exp(s_i) (fp32, Cody-Waite
  *   reduction + degree-7 polynomial, every step one rounded operation),
- *   W_i = floor(w_i * 2^40) (uint64);  candidates = the top_k heaviest by
+ *   W_i = floor(w_i * 2^24) (exact in 32 bits: the top weight is 2^24, and a
+ *   token below 2^-24 of it gets 0);  candidates = the top_k heaviest by
  *   (W desc, id asc) (top_k = 0: all);  kept = the shortest prefix of the
  *   candidates in that order with C * 2^24 >= round(top_p * 2^24) * S;
  *   r = Philox4x32-10(key = rng_seed, counter = (position of the produced
@@ -202,7 +208,9 @@ SDSAT_API sdsat_status sdsat_accept_nucleus(sdsat_ctx* ctx, sdsat_kv* kv, const 
                                   float top_p, float temperature, uint64_t rng_seed, int top_k,
                                   int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit);
 
-/* Explicit commit / rollback: len[s] = new_len_dev[s] for s < b (device values,
+/* Explicit commit / rollback (implied by Sec. 2.1.1: after Eq. 3 only the accepted
+ * prefix stays in the context; the adaptive positions of draft step 1 and the rejected
+ * drafts are dropped): len[s] = new_len_dev[s] for s < b (device values,
  * 0 <= new_len <= max_len; out-of-range values are clamped and set CAPACITY).
  * Errors: EINVAL. */
 SDSAT_API sdsat_status sdsat_kv_commit(sdsat_ctx* ctx, sdsat_kv* kv, const int32_t* new_len_dev, int b);
@@ -332,7 +340,8 @@ SDSAT_API sdsat_status sdsat_accept_pipelined(sdsat_ctx* ctx, sdsat_kv* kv, cons
                                               int32_t* accepted_len_dev, int32_t* out_tokens_dev, int commit);
 
 /* Run n prompt tokens of sequence `seq` through the model and commit them
- * (len[seq] += n): the step before the decode loop.  Chunks of up to
+ * (len[seq] += n): the step before the decode loop (Sec. 2.1.1 starts from a prompt
+ * y_1 .. y_n already in the context; the paper gives the prefill no further detail).  Chunks of up to
  * SDSAT_MAX_ROWS positions go through one block forward each (the weights stream
  * once per chunk), position i attending to every earlier position; a tail shorter
  * than SDSAT_MAX_Q rows runs as one ordinary block.  No logits are produced.
@@ -345,6 +354,9 @@ SDSAT_API sdsat_status sdsat_prefill(sdsat_ctx* ctx, sdsat_kv* kv, int seq, cons
  * ECUDA if the stream reported a CUDA error. */
 SDSAT_API sdsat_status sdsat_get_error(sdsat_ctx* ctx, uint32_t* flags);
 
+/* A static, NUL-terminated English name of a status code ("ok", "invalid argument", ...;
+ * unknown codes give "unknown status").  Host only, never fails.  The paper has no
+ * counterpart: it is the error reporting of this library's boundary. */
 SDSAT_API const char* sdsat_status_string(sdsat_status s);
 
 /* ---- single kernels (unit parity tests and kernel sweeps) ------------------------- */
@@ -407,15 +419,19 @@ SDSAT_API sdsat_status sdsat_op_exp(sdsat_ctx* ctx, const float* in_dev, float* 
  *   y_dev fp32 [M][N]; stream is a cudaStream_t (NULL = legacy default stream).
  *   Limits: 1 <= M <= 16, 8 <= K <= 16384 with K % 8 == 0, 1 <= N <= 65536;
  *   sizes past the limits return ECAPACITY, malformed arguments EINVAL.
+ *   err_dev: optional caller-owned device word (NULL: not reported); a bounded
+ *   in-kernel wait that runs out (2 s) ORs SDSAT_DEV_TIMEOUT into it and leaves
+ *   y_dev incomplete.  The call never clears it.
  * The first call on a device (with that device current) looks up the array's
  * device address and prepares the kernels; make that first call before any
- * stream capture.  Every call shares the one array: calls whose work overlaps
- * on the GPU (different streams, or concurrent host threads) race and must be
- * serialised by the caller.  The call clears the tile counters it uses; the
- * other scratch contents are overwritten before they are read.  Device-side
- * wait timeouts are not reported by this entry point.  Asynchronous on `stream`. */
+ * stream capture.  The set-up is redone when the device's context changes (after
+ * cudaDeviceReset, for instance).  Every call shares the one array: calls whose
+ * work overlaps on the GPU (different streams, or concurrent host threads) race
+ * and must be serialised by the caller.  The call clears the tile counters it
+ * uses; the other scratch contents are overwritten before they are read.
+ * Asynchronous on `stream`. */
 SDSAT_API sdsat_status sdsat_gemm_static(const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev,
-                                         void* stream);
+                                         void* stream, uint32_t* err_dev);
 
 /* ---- measurement ------------------------------------------------------------------ */
 

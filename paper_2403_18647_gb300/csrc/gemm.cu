@@ -43,9 +43,6 @@ namespace sdsat {
 #ifndef SDSAT_GEMM_STAGES16
 #define SDSAT_GEMM_STAGES16 4
 #endif
-#ifndef SDSAT_GEMM_CTAS_PER_SM
-#define SDSAT_GEMM_CTAS_PER_SM 2
-#endif
 // Minimum resident CTAs per SM the register allocation must allow (192 threads each).
 #ifndef SDSAT_GEMM_MINB
 #define SDSAT_GEMM_MINB 2
@@ -569,7 +566,7 @@ cudaError_t gemm_prepare() {
 
 static int gemm_grid(const GemmParams& p, int num_sms) {
   const long long T = (long long)p.n_tiles * p.kc;
-  const int per_sm = gemm_mpad(p.M) <= 32 ? SDSAT_GEMM_CTAS_PER_SM : 1;
+  const int per_sm = gemm_mpad(p.M) <= 32 ? GEMM_CTAS_PER_SM : 1;
   return (int)std::min<long long>((long long)num_sms * per_sm, T);
 }
 

@@ -41,6 +41,13 @@ __device__ __forceinline__ void trace_write(const Trace& t, unsigned int flags, 
 }
 
 // ---- skinny weight-streaming GEMM --------------------------------------------
+// CTAs per SM of the skinny GEMM's grid for M <= 32 (compile-time tuning; one for M > 32).
+// Every user of the grid size (the split-K partials, the fixed scratch of the
+// scratch-free entry point) sizes its buffers from this constant.
+#ifndef SDSAT_GEMM_CTAS_PER_SM
+#define SDSAT_GEMM_CTAS_PER_SM 2
+#endif
+constexpr int GEMM_CTAS_PER_SM = SDSAT_GEMM_CTAS_PER_SM;
 // Tiles of 128 output features x 64 K-elements; the 128 rows come from two
 // 64-row TMA boxes ("halves") whose source depends on the map mode.
 enum GemmMap : int {

@@ -25,8 +25,8 @@ namespace {
 constexpr int SA_MAX_M = 16;          // activation rows
 constexpr int SA_MAX_K = 16384;       // reduction length
 constexpr int SA_MAX_N = 65536;       // output features (512 tiles of 128)
-constexpr int SA_MAX_SM = 64;         // SMs used: at most 2 * 64 CTAs
-constexpr int SA_MAX_CTAS = 2 * SA_MAX_SM;
+constexpr int SA_MAX_SM = 64;         // SMs used
+constexpr int SA_MAX_CTAS = GEMM_CTAS_PER_SM * SA_MAX_SM;   // the largest grid launch_gemm builds here
 constexpr int SA_TILES = SA_MAX_N / 128;
 
 constexpr size_t SA_X_BYTES = (size_t)SA_MAX_M * SA_MAX_K * 2;          // one of hi / lo: 512 KiB
@@ -36,6 +36,10 @@ constexpr size_t SA_OFF_XLO = SA_X_BYTES;
 constexpr size_t SA_OFF_PART = 2 * SA_X_BYTES;
 constexpr size_t SA_OFF_CNT = SA_OFF_PART + SA_PART_BYTES;
 constexpr size_t SA_BYTES = SA_OFF_CNT + SA_CNT_BYTES;                   // 3 MiB + 2 KiB
+
+// the kernel writes partials [(cta * 2 + slot) * 16 rows][128] for cta < its grid
+static_assert(SA_PART_BYTES >= (size_t)SA_MAX_CTAS * 2 * 16 * 128 * sizeof(float), "partials region too small");
+static_assert(SA_OFF_CNT % 16 == 0 && SA_OFF_PART % 16 == 0, "scratch regions 16-byte aligned");
 
 }  // namespace
 }  // namespace sdsat
@@ -48,37 +52,52 @@ namespace {
 
 struct DeviceSetup {
   bool done = false;
-  unsigned char* scratch = nullptr;   // device address of g_gemm_static_scratch on this device
+  CUcontext cuctx = nullptr;          // the context the set-up was made in
+  unsigned char* scratch = nullptr;   // device address of g_gemm_static_scratch in that context
   int sms = 0;
 };
 constexpr int SA_MAX_DEVICES = 64;
 DeviceSetup g_setup[SA_MAX_DEVICES];
 std::mutex g_setup_mutex;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_static = nullptr;
+PFN_cuCtxGetCurrent_v4000 g_ctx_current = nullptr;
+
+template <typename F>
+bool driver_entry(const char* name, int version, F* fn) {
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &p, version, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !p)
+    return false;
+  *fn = reinterpret_cast<F>(p);
+  return true;
+}
 
 // Per-device set-up, done by the first call on each device (with that device
 // current): the device address of the scratch array, the SM count, the kernels'
 // shared-memory limits and the tensor-map encoder.  Host code must not use the
 // array's name as an address; it is a host-side stand-in for the device symbol.
+// The set-up belongs to the device's current context: after a cudaDeviceReset the
+// device gets a new primary context, whose scratch address and kernel attributes
+// are looked up again on the next call.
 sdsat_status setup_device(int dev, DeviceSetup** out) {
   if (dev < 0 || dev >= SA_MAX_DEVICES) return SDSAT_EUNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_setup_mutex);
+  if (!g_ctx_current && !driver_entry("cuCtxGetCurrent", 4000, &g_ctx_current)) return SDSAT_ECUDA;
+  CUcontext cur = nullptr;   // null before the runtime has made a context current on this thread
+  if (g_ctx_current(&cur) != CUDA_SUCCESS) return SDSAT_ECUDA;
   DeviceSetup& s = g_setup[dev];
-  if (!s.done) {
+  if (!s.done || !cur || s.cuctx != cur) {
+    s.done = false;
     void* ptr = nullptr;
     if (cudaGetSymbolAddress(&ptr, g_gemm_static_scratch) != cudaSuccess || ptr == nullptr) return SDSAT_ECUDA;
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return SDSAT_ECUDA;
     if (gemm_prepare() != cudaSuccess) return SDSAT_ECUDA;
-    if (!g_encode_static) {
-      void* fn = nullptr;
-      cudaDriverEntryPointQueryResult q;
-      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
-              cudaSuccess ||
-          q != cudaDriverEntryPointSuccess)
-        return SDSAT_ECUDA;
-      g_encode_static = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
+    if (!g_encode_static && !driver_entry("cuTensorMapEncodeTiled", 12000, &g_encode_static)) return SDSAT_ECUDA;
+    // the symbol lookup above made the device's context current if none was
+    if (g_ctx_current(&cur) != CUDA_SUCCESS || !cur) return SDSAT_ECUDA;
+    s.cuctx = cur;
     s.scratch = static_cast<unsigned char*>(ptr);
     s.sms = std::min(sms, SA_MAX_SM);
     s.done = true;
@@ -106,7 +125,7 @@ bool aligned16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15
 using namespace sdsat;
 
 extern "C" sdsat_status sdsat_gemm_static(const float* x_dev, int M, int K, const void* w_dev, int N, float* y_dev,
-                                          void* stream) {
+                                          void* stream, uint32_t* err_dev) {
   if (!x_dev || !y_dev || !aligned16(x_dev) || !aligned16(w_dev) || M < 1 || K < 8 || K % 8 || N < 1)
     return SDSAT_EINVAL;
   if (M > SA_MAX_M || K > SA_MAX_K || N > SA_MAX_N) return SDSAT_ECAPACITY;
@@ -137,7 +156,7 @@ extern "C" sdsat_status sdsat_gemm_static(const float* x_dev, int M, int K, cons
   g.out_ld = N;
   g.partials = partials;
   g.counters = counters;
-  g.err = nullptr;
+  g.err = err_dev;   // caller-owned; a bounded wait that runs out ORs SDSAT_DEV_TIMEOUT into it
   // the tile counters must start at zero (the kernel also leaves them at zero)
   if (cudaMemsetAsync(counters, 0, (size_t)g.n_tiles * sizeof(int), cs) != cudaSuccess) return SDSAT_ECUDA;
   if (launch_split(x_dev, M, K, xhi, xlo, cs, false) != cudaSuccess) return SDSAT_ECUDA;

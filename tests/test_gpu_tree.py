@@ -15,6 +15,7 @@ import pytest
 import torch
 
 import synth
+from nucleus_flips import flip_explained
 from oracle import decode as OD
 from oracle import model as OM
 from oracle import sampling as OS
@@ -256,7 +257,12 @@ def test_tree_loop_teacher_forced(sd, tiny, temperature):
         if st.mode == "draft":
             for j in range(q):
                 if tg[j] != st.targets[j]:
-                    assert OS.top2_gap(st.logits[j]) < TIE_GAP or sp.temperature > 0
+                    if sp.temperature > 0:
+                        ok, info = flip_explained(st.logits[j], lg[j], sp.temperature, sp.top_p, sp.top_k,
+                                                  sp.seed, st.len_before + j + 1, 0)
+                        assert ok, (j, info)
+                    else:
+                        assert OS.top2_gap(st.logits[j]) < TIE_GAP
                     flips += 1
         else:
             # the acceptance is bit-exact on the logits the GPU produced
@@ -264,12 +270,25 @@ def test_tree_loop_teacher_forced(sd, tiny, temperature):
             p_ref = OT.tree_verify(t, st.tokens, parent)
             assert acc.item() == len(p_ref)
             assert path.cpu().tolist()[:len(p_ref)] == p_ref
-            if t != list(st.targets):
-                flips += 1
-            elif flips == 0:
+            depth = OT.depths(parent)
+            step_flips = 0
+            for j in range(q):
+                if t[j] != st.targets[j]:
+                    if sp.temperature > 0:
+                        ok, info = flip_explained(st.logits[j], lg[j], sp.temperature, sp.top_p, sp.top_k,
+                                                  sp.seed, st.len_before + depth[j] + 1, 0)
+                        assert ok, (j, info)
+                    else:
+                        assert OS.top2_gap(st.logits[j]) < TIE_GAP
+                    step_flips += 1
+            if step_flips == 0 and flips == 0:
                 assert acc.item() == st.accepted
+            flips += step_flips
     assert n_tree_steps >= 5
-    assert flips <= (1 if temperature == 0 else len(res.steps))
+    # greedy: at most one near-tie; a sampled target differs only where its row's logit error
+    # can move a sampling boundary across the shared draw (checked row by row above)
+    n_rows = sum(len(st.tokens) for st in res.steps)
+    assert flips <= (1 if temperature == 0 else n_rows // 4), (flips, n_rows)
     assert ctx.get_error() == 0
 
 
