@@ -59,17 +59,15 @@ WORKLOADS = {
 
 
 # DRAM bytes (read + write) per algorithmic byte of the skinny GEMM, from one ncu capture
-# (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.57 MB of traffic for
-# 181.0 MB of weights + operand + output.  Applied to the average launch of the step.
-# GEMM_TRAFFIC_CURRENT says whether that capture was taken of the kernel as it is now: the
-# kernel has changed since (the epilogue warps' timeout decision became one AND-reduction
-# barrier; no memory access changed), so the bench line reports traffic null and the last
-# capture beside it until the kernel is captured again.
-GEMM_TRAFFIC_RATIO = 186.57 / 181.0
+# (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.13 MB of traffic for
+# 180.98 MB of weights + operand + output.  The bench line applies it to the step's gate/up
+# launch (the roofline's kernel).  GEMM_TRAFFIC_CURRENT says whether that capture was taken of
+# the kernel as it is now; while it is False the line reports traffic null.
+GEMM_TRAFFIC_RATIO = 186.13 / 180.98
 GEMM_TRAFFIC_CURRENT = False
-GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.57 MB for 181.0 MB "
-                       "algorithmic, profiles/gemm_gateup_4096x22016_m6.md), ratio scaled to the average launch; "
-                       "bytes per launch")
+GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.13 MB for 180.98 MB "
+                       "algorithmic, profiles/gemm_gateup_4096x22016_m6.md) times the gate/up launch's algorithmic "
+                       "bytes; bytes per launch")
 
 
 def expected_tokens_per_step(k: int, match: float, matches=None) -> float:
@@ -566,6 +564,11 @@ def run_ours(args, wl, rank, world):
     g_launches = sum(kstats.get(n, (0, 0))[0] for n in gb)
     peak, peak_kind = peaks()
     achieved = g_bytes / (g_ms / 1e3) / 1e9 if g_ms > 0 else 0.0
+    # the launch with the largest share of the step's device time: gate/up
+    gu_n, gu_ms = kstats.get("gemm_gateup", (0, 0.0))
+    gu_bytes = gb["gemm_gateup"]
+    gu_achieved = gu_bytes / (gu_ms / gu_n / 1e3) / 1e9 if gu_n and gu_ms > 0 else 0.0
+    prof_ms = sum(v[1] for v in kstats.values())
     # per-step algorithmic bytes over one calibrated generation
     Wb = weight_bytes(shape)
     slot = kv_bytes_per_layer_slot(shape) * shape.n_layers
@@ -610,17 +613,21 @@ def run_ours(args, wl, rank, world):
         "step_hbm": {"bytes": int(step_bytes), "achieved_gbs": round(step_gbs, 1),
                      "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4),
                      "frac_of_measured": round(step_gbs / peak, 4)},
-        "roofline": {"kernel": "skinny_gemm (all projections)", "bound": "hbm", "achieved": round(achieved, 1),
-                     "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "traffic": (int(GEMM_TRAFFIC_RATIO * g_bytes / max(1, g_launches))
-                                 if GEMM_TRAFFIC_CURRENT else None),
-                     "traffic_source": GEMM_TRAFFIC_SOURCE,
-                     "traffic_last_capture": {"bytes_per_launch": int(GEMM_TRAFFIC_RATIO * g_bytes / max(1, g_launches)),
-                                              "ratio_to_algorithmic": round(GEMM_TRAFFIC_RATIO, 4),
-                                              "current": GEMM_TRAFFIC_CURRENT},
-                     "peak_source": peak_kind, "launches": g_launches,
-                     "bytes_per_launch": int(g_bytes / max(1, g_launches)),
-                     "ms_per_launch": round(g_ms / max(1, g_launches), 5)},
+        "roofline": {"kernel": "gemm_kernel, gate/up launch (K %d, N %d, M %s)" %
+                               (shape.d_model, 2 * shape.ffn_dim, "/".join(str(m) for m in sorted({r.b * r.q, r.b * r.q2}))),
+                     "bound": "hbm", "achieved": round(gu_achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(gu_achieved / peak, 4),
+                     "traffic": int(GEMM_TRAFFIC_RATIO * gu_bytes) if GEMM_TRAFFIC_CURRENT else None,
+                     "traffic_source": GEMM_TRAFFIC_SOURCE, "peak_source": peak_kind,
+                     "bytes_per_launch": int(gu_bytes), "ms_per_launch": round(gu_ms / max(1, gu_n), 5),
+                     "launches": gu_n, "share_of_profiled_step": round(gu_ms / max(1e-9, prof_ms), 4),
+                     "timing": "profiled pass: CUDA events around every launch on the context stream, so launches "
+                               "are serialised (no programmatic dependent launch overlap): %.3f ms per step there "
+                               "against %.3f ms graph-replayed; per-kernel fractions are lower bounds" %
+                               (prof_ms / n_prof, ms_step),
+                     "all_gemm": {"achieved": round(achieved, 1), "frac": round(achieved / peak, 4),
+                                  "launches": g_launches, "bytes_per_launch": int(g_bytes / max(1, g_launches)),
+                                  "ms_per_launch": round(g_ms / max(1, g_launches), 5)}},
         "kernels": {k: {"launches": v[0], "ms_total": round(v[1], 4), "us_per_launch": round(1e3 * v[1] / v[0], 2)}
                     for k, v in kstats.items()},
         "e2e": e2e, "gpu_launches": gpu_launches, "device_error_flags": flags,
@@ -984,6 +991,17 @@ def run_ksweep(args):
         torch.cuda.synchronize()
 
 
+def kernel_us(ctx, name, reps, call):
+    """Mean device time of one launch of kernel class `name` over `reps` calls, from the
+    library's profiling hook (CUDA events around each launch)."""
+    ctx.profile_begin(2 * reps + 16)
+    for i in range(reps):
+        call(i)
+    st = ctx.profile_end()
+    n, ms = st.get(name, (0, 0.0))
+    return 1e3 * ms / n if n else float("nan")
+
+
 def run_sweep(args):
     """Kernel sweeps on 7B shapes (one JSON line per case): the skinny GEMM with M = q against
     bf16 weights, and block-causal attention of q rows (32 heads x 128) against a bf16 cache.
@@ -1016,11 +1034,15 @@ def run_sweep(args):
                 e1.record()
                 torch.cuda.synchronize()
                 us = e0.elapsed_time(e1) * 1e3 / reps
+                kus = kernel_us(ctx, "gemm_op", reps, lambda i: ctx.op_gemm(x, ws[i % nbuf], y))
                 by = K * N * 2 + M * K * 4 + M * N * 4
                 cases.append({"kernel": "skinny_gemm", "M": M, "K": K, "N": N, "us": round(us, 2),
                               "GB/s": round(by / us / 1e3, 1), "frac_of_measured": round(by / us / 1e3 / peak, 4),
                               "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4),
-                              "note": "includes the fp32 -> bf16 hi/lo operand split kernel"})
+                              "kernel_us": round(kus, 2), "kernel_GB/s": round(by / kus / 1e3, 1),
+                              "kernel_frac_of_measured": round(by / kus / 1e3 / peak, 4),
+                              "note": "us: back-to-back calls, each with the fp32 -> bf16 hi/lo operand split kernel; "
+                                      "kernel_us: the GEMM kernel alone (CUDA events around each launch)"})
             del ws
     if args.sweep in ("attention", "all"):
         H, hd = 32, 128
@@ -1045,11 +1067,15 @@ def run_sweep(args):
                 e1.record()
                 torch.cuda.synchronize()
                 us = e0.elapsed_time(e1) * 1e3 / reps
+                kus = kernel_us(ctx, "attention_op", reps,
+                                lambda i: ctx.op_attention(Q, Ks[i % nbuf], Vs[i % nbuf], ln, 1, q, H, hd, cap, out))
                 by = 2 * H * (n + q) * hd * 2 + 2 * q * H * hd * 4
                 cases.append({"kernel": "attention", "q": q, "ctx": n, "heads": H, "head_dim": hd,
                               "us": round(us, 2), "GB/s": round(by / us / 1e3, 1),
                               "frac_of_measured": round(by / us / 1e3 / peak, 4),
-                              "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4)})
+                              "frac_of_8tbs": round(by / us / 1e3 / NOMINAL_HBM_GBS, 4),
+                              "kernel_us": round(kus, 2), "kernel_GB/s": round(by / kus / 1e3, 1),
+                              "kernel_frac_of_measured": round(by / kus / 1e3 / peak, 4)})
             del Ks, Vs
     if args.sweep in ("prefill", "all"):
         # the prefill path's tiled GEMM (M positions x the 7B projections), tensor-core bound

@@ -184,17 +184,18 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
 #pragma unroll
   for (int m = 0; m < MPAD; ++m) staging[r * (MPAD + 1) + m] = acc[m];
   named_bar_sync(1, 128);
+  // These epilogues run once per launch, on the tiles' reducers, so their instructions are
+  // fetched cold: the row loops stay rolled (a few dozen instructions) and read the
+  // accumulators back from the exchange area instead of unrolling over MPAD rows.
+  const float* mine = staging + r * (MPAD + 1);
   if (p.epi == EPI_SWIGLU) {
     const int j = 64 * tile + r;
     if (r < 64 && j < p.N) {
-      // the up projections (lanes 64-127) leave shared memory before any store is issued
-#pragma unroll
-      for (int m = 0; m < MPAD; ++m)
-        if (m < M) acc[m] = acc[m] / (1.0f + expf(-acc[m])) * staging[(r + 64) * (MPAD + 1) + m];
-#pragma unroll
-      for (int m = 0; m < MPAD; ++m) {
-        if (m >= M) break;
-        const float a = acc[m];
+      const float* up = staging + (r + 64) * (MPAD + 1);   // the up projection, lane r + 64
+#pragma unroll 1
+      for (int m = 0; m < M; ++m) {
+        const float g = mine[m];
+        const float a = g / (1.0f + expf(-g)) * up[m];
         p.out[(size_t)m * p.out_ld + j] = a;
         const __nv_bfloat16 hi = __float2bfloat16_rn(a);
         p.out_hi[(size_t)m * p.out_ld + j] = hi;
@@ -209,36 +210,23 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int hd = p.hd, half = hd >> 1;
     const int head = f / hd, i = f % hd;
     const int partner = (i < half) ? r + half : r - half;
-#pragma unroll
-    for (int m0 = 0; m0 < MPAD; m0 += EG) {
-      // a group's rotated values first, then its stores (shared-memory reads queue behind stores)
-      int slot[EG];
-      float val[EG];
-#pragma unroll
-      for (int u = 0; u < EG; ++u) {
-        const int m = m0 + u;
-        slot[u] = 0;
-        val[u] = 0.f;
-        if (m < M) {
-          slot[u] = s_slot[m];
-          val[u] = acc[m];
-          if (which < 2) {   // rotate-half RoPE with the partner lane's value from shared memory
-            const float2 cs = s_cs[m * 64 + (i % half)];
-            const float y = staging[partner * (MPAD + 1) + m];
-            val[u] = (i < half) ? acc[m] * cs.x - y * cs.y : acc[m] * cs.x + y * cs.y;
-          }
-        }
+    const float* other = staging + partner * (MPAD + 1);
+    const float sgn = (i < half) ? -1.f : 1.f;   // rotate-half RoPE: x cos -+ partner sin
+    __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
+#pragma unroll 1
+    for (int m = 0; m < M; ++m) {
+      float val = mine[m];
+      if (which < 2) {
+        const float2 cs = s_cs[m * 64 + (i % half)];
+        val = val * cs.x + sgn * (other[m] * cs.y);
       }
-#pragma unroll
-      for (int u = 0; u < EG; ++u) {
-        const int m = m0 + u;
-        if (m >= M) break;
-        const int s = p.seq0 + m / p.q;
-        if (which == 0) {
-          p.out[(size_t)m * p.out_ld + f] = val[u];
-        } else if (slot[u] < p.cap) {
-          __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
-          cache[(((size_t)s * p.H + head) * p.cap + slot[u]) * hd + i] = __float2bfloat16_rn(val[u]);
+      if (which == 0) {
+        p.out[(size_t)m * p.out_ld + f] = val;
+      } else {
+        const int slot = s_slot[m];
+        if (slot < p.cap) {
+          const int s = p.seq0 + m / p.q;
+          cache[(((size_t)s * p.H + head) * p.cap + slot) * hd + i] = __float2bfloat16_rn(val);
         } else if (i == 0 && which == 1) {
           set_error(p.err, ERR_CAPACITY);
         }
