@@ -49,7 +49,7 @@ namespace sdsat {
 #endif
 // Epilogue rows handled per group: a group's loads are all issued before its stores.
 #ifndef SDSAT_GEMM_EPI_GROUP
-#define SDSAT_GEMM_EPI_GROUP 8
+#define SDSAT_GEMM_EPI_GROUP 16
 #endif
 constexpr int EG = SDSAT_GEMM_EPI_GROUP;
 
