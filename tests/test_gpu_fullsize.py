@@ -241,3 +241,88 @@ def test_13b_greedy_full_size(sd):
     wts = Weights(sd, "13b", max_position=4096 + 64, cache_weights=False)
     f1, f2 = _two_step(Model(wts, 1, 4096), OD.SamplingParams(), [4], tag=13)
     assert f1 + f2 <= 1
+
+
+def _i32(v):
+    return torch.tensor(v, dtype=torch.int32, device="cuda")
+
+
+def test_7b_tree_full_size(weights_7b):
+    """The tree-structured draft step 2 (Sec. 2.1.2) at the 7B shape, every layer: two chains of
+    k = 5 drafts below the root (q = 11), tree attention mask and depth-based RoPE positions.
+    Branch 0 is wrong at depth 1, branch 1 copies the plain greedy continuation to depth 3, so
+    the longest accepted branch is [0, 6, 7, 8].  Logits, targets and the path are compared with
+    the oracle, and the K / V rows the GPU moved to contiguous slots with the oracle's commit."""
+    from oracle import tree as OT
+    m = Model(weights_7b, 1, 2048)
+    shape, L0 = m.shape, m.ctx_len
+    sp = OD.SamplingParams()
+    root = int(synth.uniform_ids(21, 0, 1, shape.adaptive_id)[0])
+    g = OD.plain_decode(m.W, m.kvo, 0, root, K, sp)   # the plain continuation after the root
+    m.set_len([L0])
+    wrong = [(x + 1) % shape.vocab for x in g]
+    drafts = [[wrong[0]] + g[1:K], g[:3] + wrong[3:K]]
+    parent = OT.chains_parent(2, K)
+    q2 = len(parent)
+    toks = [root] + drafts[0] + drafts[1]
+    lt = torch.empty(q2, shape.vocab, device="cuda")
+    acc = torch.empty(1, dtype=torch.int32, device="cuda")
+    out = torch.empty(q2, dtype=torch.int32, device="cuda")
+    path = torch.empty(q2, dtype=torch.int32, device="cuda")
+    m.ctx.block_forward_tree(m.kv, _i32(toks), _i32(parent), lt, 1, q2)
+    m.ctx.accept_tree(m.kv, lt, _i32(toks), _i32(parent), 1, q2, acc, out, path)
+    lg = lt.cpu().numpy().astype(np.float64)
+    assert m.ctx.get_error() == 0
+    ref = OT.tree_forward(m.W, m.kvo, 0, toks, parent)
+    _compare_logits(lg, ref)
+    t_ref = OT.tree_targets(ref, sp, parent, L0, 0)
+    t_gpu = OT.tree_targets(lg, sp, parent, L0, 0)
+    flips = [j for j in range(q2) if t_ref[j] != t_gpu[j]]
+    assert all(OS.top2_gap(ref[j]) < TIE_GAP for j in flips), flips
+    p_ref = OT.tree_verify(t_ref, toks, parent)
+    if not flips:
+        assert p_ref == [0, 6, 7, 8]
+        assert path.cpu().tolist()[:len(p_ref)] == p_ref and int(acc.item()) == len(p_ref)
+        assert out.cpu().tolist()[:len(p_ref)] == [t_ref[n] for n in p_ref]
+    # the accepted branch's K / V rows, moved to slots L0 + 1 .. L0 + m on both sides
+    OT.tree_commit(m.kvo, 0, p_ref)
+    assert m.ctx.kv_lengths(m.kv).item() == L0 + len(p_ref)
+    for l in (0, shape.n_layers - 1):
+        k, v = m.ctx.kv_read(m.kv, l, 0, L0, len(p_ref))
+        for got, want in ((k, m.kvo.K[l][0][:, L0:L0 + len(p_ref)]), (v, m.kvo.V[l][0][:, L0:L0 + len(p_ref)])):
+            err = np.abs(got.float().cpu().numpy() - want)
+            assert (err <= 2.0 ** -7 * np.abs(want) + 1e-3).all(), (l, err.max())
+
+
+def test_7b_pipelined_block_full_size(weights_7b):
+    """The pipelined variant's mode-A block at the 7B shape (q = 2k + 1 = 11 rows: x_0, k drafts,
+    k adaptive tokens), every layer: drafts copy the plain greedy continuation to depth 2, so Eq. 3
+    accepts 2 of them.  Logits, targets and the accepted count against the oracle."""
+    m = Model(weights_7b, 1, 2048)
+    shape, L0 = m.shape, m.ctx_len
+    sp = OD.SamplingParams()
+    x0 = int(synth.uniform_ids(22, 0, 1, shape.adaptive_id)[0])
+    g = OD.plain_decode(m.W, m.kvo, 0, x0, 3, sp)
+    m.set_len([L0])
+    drafts = g[:2] + [(g[2] + 1) % shape.vocab] + synth.uniform_ids(22, 1, K - 3, shape.vocab).tolist()
+    blk = [x0] + drafts + [shape.adaptive_id] * K
+    q = len(blk)
+    logits = torch.empty(q, shape.vocab, device="cuda")
+    acc = torch.empty(1, dtype=torch.int32, device="cuda")
+    out = torch.empty(q, dtype=torch.int32, device="cuda")
+    m.ctx.block_forward(m.kv, _i32(blk), logits, 1, q)
+    m.ctx.accept_pipelined(m.kv, logits, _i32(blk), _i32([K]), 1, q, acc, out)
+    lg = logits.cpu().numpy().astype(np.float64)
+    assert m.ctx.get_error() == 0
+    ref = OM.block_forward(m.W, m.kvo, 0, blk)
+    _compare_logits(lg, ref)
+    t_ref, _ = OD.row_targets(ref, sp, L0 + 1, 0)
+    t_gpu, _ = OD.row_targets(lg, sp, L0 + 1, 0)
+    assert out.cpu().tolist()[:int(acc.item())] == t_gpu[:int(acc.item())]
+    flips = [j for j in range(q) if t_ref[j] != t_gpu[j]]
+    assert all(OS.top2_gap(ref[j]) < TIE_GAP for j in flips), flips
+    m_ref = OD.verify(t_ref, blk, K)
+    assert m_ref == 2
+    if not flips:
+        assert int(acc.item()) == 1 + m_ref
+        assert t_ref[:m_ref + 1] == g[:m_ref + 1]
