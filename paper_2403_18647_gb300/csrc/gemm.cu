@@ -304,19 +304,27 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
       constexpr uint32_t TX = C::W_BYTES + 2 * C::X_BYTES;
       const long long n = g1 - g0;
       const int npre = (int)std::min<long long>(S, n);
-      auto load_w = [&](int it) {
-        const long long g = g0 + it;
-        const int tile = (int)(g / p.kc), kc = (int)(g % p.kc);
+      // This thread's per-unit work sits on the streaming path (a stage is refilled only after
+      // it has issued the copies), so the next unit's (tile, chunk) and its tile's two box
+      // sources are advanced incrementally: no division per unit.
+      int w_tile = (int)(g0 / p.kc), w_kc = (int)(g0 % p.kc), x_kc = w_kc;
+      int map0, row0, map1, row1;
+      tile_half_src(p.map_mode, p.rows_per_map, w_tile, 0, map0, row0);
+      tile_half_src(p.map_mode, p.rows_per_map, w_tile, 1, map1, row1);
+      auto load_w = [&](int it) {   // units in order, one call each
         uint8_t* dst = stages + (size_t)(it % S) * C::STAGE_BYTES;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          int map, row;
-          tile_half_src(p.map_mode, p.rows_per_map, tile, h, map, row);
-          tma_load_2d(dst + h * 8192, &p.tmap[map], &full[it % S], kc * 64, row, pol_w);
+        tma_load_2d(dst, &p.tmap[map0], &full[it % S], w_kc * 64, row0, pol_w);
+        tma_load_2d(dst + 8192, &p.tmap[map1], &full[it % S], w_kc * 64, row1, pol_w);
+        if (++w_kc == p.kc) {
+          w_kc = 0;
+          ++w_tile;
+          tile_half_src(p.map_mode, p.rows_per_map, w_tile, 0, map0, row0);
+          tile_half_src(p.map_mode, p.rows_per_map, w_tile, 1, map1, row1);
         }
       };
-      auto load_x = [&](int it) {
-        const int kc = (int)((g0 + it) % p.kc);
+      auto load_x = [&](int it) {   // units in order, one call each
+        const int kc = x_kc;
+        if (++x_kc == p.kc) x_kc = 0;
         uint8_t* dst = stages + (size_t)(it % S) * C::STAGE_BYTES + C::W_BYTES;
         tma_load_2d(dst, &p.tmap_x[0], &full[it % S], kc * 64, 0, pol_x);
         tma_load_2d(dst + C::X_BYTES, &p.tmap_x[1], &full[it % S], kc * 64, 0, pol_x);
