@@ -44,6 +44,14 @@ namespace sdsat {
 #define SDSAT_GEMM_STAGES16 4
 #endif
 // Minimum resident CTAs per SM the register allocation must allow (192 threads each).
+// Stream-K split points within the first SDSAT_GEMM_SNAP units of a tile move to the tile's
+// start, for GEMMs with at least SDSAT_GEMM_SNAP_MIN_UNITS units per CTA.
+#ifndef SDSAT_GEMM_SNAP
+#define SDSAT_GEMM_SNAP 3
+#endif
+#ifndef SDSAT_GEMM_SNAP_MIN_UNITS
+#define SDSAT_GEMM_SNAP_MIN_UNITS 24
+#endif
 #ifndef SDSAT_GEMM_MINB
 #define SDSAT_GEMM_MINB 2
 #endif
@@ -65,11 +73,29 @@ struct GemmCfg {
   static constexpr int NBAR = 2 * STAGES + 6;
   static constexpr int CS = MPAD * 64;           // EPI_QKV: RoPE (cos, sin) of every row and frequency
   static constexpr size_t SMEM =
-      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + CS * 8 + NBAR * 8 + 64;
+      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + CS * 8 + NBAR * 8 + 128;
 };
 
-__device__ __forceinline__ long long cta_of_chunk(long long g, long long T, int P) {
-  return ((g + 1) * P - 1) / T;
+// First unit of CTA b's range.  The even split b*T/P moves back to the start of its tile
+// when it falls within that tile's first `snap` units: CTA b-1 would otherwise end with a
+// segment of a few units, whose epilogue waits behind the publication (or the reduction) of
+// the CTA's first tile and so usually arrives last and reduces that tile late.  The units go
+// to CTA b instead, at the start of its range.
+// (32-bit arithmetic: the host keeps T * P below 2^31.)
+__device__ __forceinline__ int unit_begin(int b, int T, int P, int kc, int snap) {
+  int x = (int)((unsigned)b * (unsigned)T / (unsigned)P);
+  if (b > 0 && b < P) {
+    const int r = x % kc;
+    if (r >= 1 && r <= snap) x -= r;
+  }
+  return x;
+}
+
+// The CTA whose range holds unit g.  Without snapping it is the largest b with b*T/P <= g;
+// snapping moves split points back by at most snap < T/P units, so it is that b or b + 1.
+__device__ __forceinline__ int cta_of_chunk(int g, int T, int P, int kc, int snap) {
+  const int b = (int)(((unsigned)g * (unsigned)P + (unsigned)(P - 1)) / (unsigned)T);
+  return (b + 1 < P && unit_begin(b + 1, T, P, kc, snap) <= g) ? b + 1 : b;
 }
 
 // (tensor map, first row) of half h (0: tile rows 0-63, 1: rows 64-127) of tile t
@@ -260,13 +286,15 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   int* s_last = reinterpret_cast<int*>(tmem_slot + 2);
   // trace marks: first MMA issued, last accumulator ready, last tile reduced; [3] = flags
   unsigned long long* s_mark = reinterpret_cast<unsigned long long*>(tmem_slot + 4);
+  int* s_share = reinterpret_cast<int*>(s_mark + 4);   // [6] split-K bookkeeping (see the epilogue)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int cta = blockIdx.x;
-  const long long T = (long long)p.n_tiles * p.kc;
+  const int T = p.n_tiles * p.kc;
   const unsigned long long t_entry = p.trace.rec ? globaltimer_ns() : 0;
   unsigned long long t_wait = 0;
-  const long long g0 = (long long)cta * T / p.P, g1 = (long long)(cta + 1) * T / p.P;
+  const long long g0 = unit_begin(cta, T, p.P, p.kc, p.snap), g1 = unit_begin(cta + 1, T, p.P, p.kc, p.snap);
+  const int tile_first = (int)g0 / p.kc, tile_last = ((int)g1 - 1) / p.kc;
 
   if (threadIdx.x == 64) {   // the tensor maps into the TMA unit while the CTA sets up
     const int nmaps = p.map_mode == MAP_QKV3 ? 3 : (p.map_mode == MAP_GATEUP ? 2 : 1);
@@ -353,11 +381,11 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
     // ------------------------------------------------ tensor-core issue
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * MPAD);
-      int it = 0, seg = 0;
+      int it = 0, seg = 0, tile = tile_first - 1;
       long long g = g0;
       bool ok = true;
       while (ok && g < g1) {
-        const int tile = (int)(g / p.kc);
+        ++tile;   // segments are consecutive tiles
         const long long gend = std::min(g1, (long long)(tile + 1) * p.kc);
         const int buf = seg & 1;
         if (!mbar_wait_bounded(&acc_empty[buf], ((seg >> 1) & 1) ^ 1, abort_flag, p.err)) break;
@@ -423,10 +451,27 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         s_cs[(i / half) * 64 + i % half] = p.rope[(size_t)s_pos[i / half] * half + i % half];
       named_bar_sync(1, 128);
     }
-    int seg = 0;
+    // Split-K bookkeeping of the only tiles this CTA can share, its first and its last: their
+    // contributors lo..hi, and the partial slot of lo (0 when lo's range starts at the tile's
+    // start, else 1).  Every later contributor's range starts inside the tile, so its partial
+    // sits in slot 0.  Worked out once, here, into shared memory (read after the accumulator
+    // barrier): the reduction at the CTA's end is latency-bound and these divisions would sit
+    // on its path, and six values live in registers through the epilogue cost more registers
+    // than the next kernel's early CTAs can spare.
+    if (r == 0) {
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int t = i ? tile_last : tile_first;
+        const int lo = cta_of_chunk(t * p.kc, T, p.P, p.kc, p.snap);
+        s_share[3 * i] = lo;
+        s_share[3 * i + 1] = cta_of_chunk(t * p.kc + p.kc - 1, T, p.P, p.kc, p.snap);
+        s_share[3 * i + 2] = unit_begin(lo, T, p.P, p.kc, p.snap) == t * p.kc ? 0 : 1;
+      }
+    }
+    int seg = 0, tile = tile_first - 1;
     long long g = g0;
     while (g < g1) {
-      const int tile = (int)(g / p.kc);
+      ++tile;   // segments are consecutive tiles
       g = std::min(g1, (long long)(tile + 1) * p.kc);
       const int buf = seg & 1;
       // what this tile's epilogue reads from global memory (first row group), loaded while
@@ -462,13 +507,14 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
       ++seg;
 
-      const long long tstart = (long long)tile * p.kc;
-      const int c_lo = (int)cta_of_chunk(tstart, T, p.P);
-      const int c_hi = (int)cta_of_chunk(tstart + p.kc - 1, T, p.P);
+      // contributors of this tile (a tile between the first and the last is the CTA's alone)
+      const int sh = tile == tile_first ? 0 : 3;
+      const bool edge = tile == tile_first || tile == tile_last;
+      const int c_lo = edge ? s_share[sh] : cta, c_hi = edge ? s_share[sh + 1] : cta;
+      const int lo_slot = s_share[sh + 2];
       if (c_hi > c_lo) {
         // this tile is shared: publish the partial, the last contributor reduces
-        const int my_first_tile = (int)(g0 / p.kc);
-        const int slot = (tile == my_first_tile) ? 0 : 1;
+        const int slot = (tile == tile_first) ? 0 : 1;
         float* mine = p.partials + (size_t)(cta * 2 + slot) * MPAD * 128;
 #pragma unroll
         for (int m = 0; m < MPAD; ++m)
@@ -499,10 +545,9 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
             named_bar_sync(1, 128);   // the previous round's shared-memory reads are done; bytes announced
             if (r < cnt) {            // one copy per thread
               const int j = j0 + r;
-              const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
               fence_proxy_async_global();
               bulk_load_g2s(stages + (size_t)r * pbytes,
-                            p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128, pbytes, red_bar);
+                            p.partials + (size_t)(j * 2 + (j == c_lo ? lo_slot : 0)) * MPAD * 128, pbytes, red_bar);
             }
             ok = named_bar_and(1, 128, mbar_wait_bounded(red_bar, ph, abort_flag, p.err));
             ph ^= 1u;
@@ -519,8 +564,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
           if (!ok) break;
         } else {
           for (int j = c_lo; j <= c_hi; ++j) {
-            const int jfirst = (int)(((long long)j * T / p.P) / p.kc);
-            const float* src = p.partials + (size_t)(j * 2 + (tile == jfirst ? 0 : 1)) * MPAD * 128;
+            const float* src = p.partials + (size_t)(j * 2 + (j == c_lo ? lo_slot : 0)) * MPAD * 128;
 #pragma unroll
             for (int m = 0; m < MPAD; ++m)
               if (m < p.M) acc[m] += __ldcg(src + m * 128 + r);
@@ -569,6 +613,11 @@ static int gemm_grid(const GemmParams& p, int num_sms) {
 cudaError_t launch_gemm(GemmParams& p, int num_sms, cudaStream_t st, bool pdl) {
   const int mpad = gemm_mpad(p.M);
   p.P = gemm_grid(p, num_sms);
+  if ((long long)p.n_tiles * p.kc * p.P >= (1LL << 31)) return cudaErrorInvalidValue;   // 32-bit split math
+  // Snapping costs the next CTA up to `snap` units, so it is used only where a CTA's share
+  // is long; it needs snap < T/P (a range never empties and a unit's owner stays b or b+1).
+  const long long per = (long long)p.n_tiles * p.kc / p.P;
+  p.snap = per >= SDSAT_GEMM_SNAP_MIN_UNITS ? (int)std::min<long long>(SDSAT_GEMM_SNAP, per - 1) : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.P);
   cfg.blockDim = dim3(192);

@@ -72,6 +72,7 @@ struct GemmParams {
   int n_tiles;
   int kc;             // K chunks of 64
   int P;              // CTAs
+  int snap;           // stream-K split points within a tile's first `snap` units move to the tile start
   int M;              // activation rows (<= MPAD)
   // epilogue
   int epi;
