@@ -73,7 +73,7 @@ struct GemmCfg {
   static constexpr int NBAR = 2 * STAGES + 6;
   static constexpr int CS = MPAD * 64;           // EPI_QKV: RoPE (cos, sin) of every row and frequency
   static constexpr size_t SMEM =
-      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 3 * 64 * 4 + CS * 8 + NBAR * 8 + 128;
+      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 4 * 64 * 4 + CS * 8 + NBAR * 8 + 128;
 };
 
 // First unit of CTA b's range.  The even split b*T/P moves back to the start of its tile
@@ -123,8 +123,8 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 
 template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
-                                               float* staging, const float* sinv, const int* s_slot,
-                                               const int* s_pos, const float (&pre)[EG], float pre_gn,
+                                               float* staging, const float* sinv, const int* s_slot, const int* s_seq,
+                                               const float (&pre)[EG], float pre_gn,
                                                const float2* s_cs) {
   const int M = p.M;
   if (p.ssq_in) {
@@ -229,12 +229,16 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
       }
     }
   } else {  // EPI_QKV
+    // This runs once per launch on the reducers' critical path, so no division: the
+    // projection by comparison, head and dimension by shift and mask (hd is 64 or 128), and
+    // each row's sequence from the table the setup filled.
     const int R = p.rows_per_map;
     const int gf = 128 * tile + r;
-    const int which = gf / R;
-    const int f = gf % R;
+    const int which = (gf >= R) + (gf >= 2 * R);
+    const int f = gf - which * R;
     const int hd = p.hd, half = hd >> 1;
-    const int head = f / hd, i = f % hd;
+    const int head = f >> (__ffs(hd) - 1), i = f & (hd - 1);
+    const int ih = i & (half - 1);
     const int partner = (i < half) ? r + half : r - half;
     const float* other = staging + partner * (MPAD + 1);
     const float sgn = (i < half) ? -1.f : 1.f;   // rotate-half RoPE: x cos -+ partner sin
@@ -243,7 +247,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     for (int m = 0; m < M; ++m) {
       float val = mine[m];
       if (which < 2) {
-        const float2 cs = s_cs[m * 64 + (i % half)];
+        const float2 cs = s_cs[m * 64 + ih];
         val = val * cs.x + sgn * (other[m] * cs.y);
       }
       if (which == 0) {
@@ -251,7 +255,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
       } else {
         const int slot = s_slot[m];
         if (slot < p.cap) {
-          const int s = p.seq0 + m / p.q;
+          const int s = s_seq[m];
           cache[(((size_t)s * p.H + head) * p.cap + slot) * hd + i] = __float2bfloat16_rn(val);
         } else if (i == 0 && which == 1) {
           set_error(p.err, ERR_CAPACITY);
@@ -273,7 +277,8 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   float* sinv = staging + C::STAGING;   // [64] RMSNorm row factors of the operand
   int* s_slot = reinterpret_cast<int*>(sinv + 64);   // [64] EPI_QKV: cache slot of each row
   int* s_pos = s_slot + 64;                          // [64] EPI_QKV: RoPE position of each row
-  float2* s_cs = reinterpret_cast<float2*>(s_pos + 64);   // [MPAD][64] EPI_QKV: RoPE factors
+  int* s_seq = s_pos + 64;                           // [64] EPI_QKV: sequence of each row
+  float2* s_cs = reinterpret_cast<float2*>(s_seq + 64);   // [MPAD][64] EPI_QKV: RoPE factors
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_cs + C::CS);
   uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
   uint64_t* empty = bars + S;        // stage consumed by the tensor core
@@ -435,7 +440,8 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
     }
     if (p.epi == EPI_QKV) {   // cache slot and RoPE position of every row (fixed during the forward)
       if (r < p.M) {
-        const int slot = __ldcg(p.len + p.seq0 + r / p.q) + r % p.q;
+        const int seq = p.seq0 + r / p.q;
+        const int slot = __ldcg(p.len + seq) + r % p.q;
         int pos = p.positions ? __ldcg(p.positions + r) : slot;
         if (pos < 0 || pos >= p.rope_len) {
           set_error(p.err, ERR_POSITION);
@@ -443,6 +449,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         }
         s_slot[r] = slot;
         s_pos[r] = pos;
+        s_seq[r] = seq;
       }
       named_bar_sync(1, 128);
       // the RoPE factors of every row, in shared memory long before any accumulator is ready
@@ -573,7 +580,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         if (r == 0) p.counters[tile] = 0;
       }
       if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
-      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_pos, pre, pre_gn, s_cs);
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_seq, pre, pre_gn, s_cs);
     }
   }
 
