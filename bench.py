@@ -64,7 +64,7 @@ WORKLOADS = {
 # launch (the roofline's kernel).  GEMM_TRAFFIC_CURRENT says whether that capture was taken of
 # the kernel as it is now; while it is False the line reports traffic null.
 GEMM_TRAFFIC_RATIO = 186.02 / 180.98
-GEMM_TRAFFIC_CURRENT = True
+GEMM_TRAFFIC_CURRENT = False
 GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.02 MB for 180.98 MB "
                        "algorithmic, profiles/gemm_gateup_4096x22016_m6.md) times the gate/up launch's algorithmic "
                        "bytes; bytes per launch")
