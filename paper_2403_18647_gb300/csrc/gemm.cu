@@ -218,10 +218,12 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int j = 64 * tile + r;
     if (r < 64 && j < p.N) {
       const float* up = staging + (r + 64) * (MPAD + 1);   // the up projection, lane r + 64
+      // SiLU through the fast exponential and division (a few ulp, far inside the tolerances
+      // of an fp32 operand): the row loop is one dependent chain on the reducers' critical path
 #pragma unroll 1
       for (int m = 0; m < M; ++m) {
         const float g = mine[m];
-        const float a = g / (1.0f + expf(-g)) * up[m];
+        const float a = __fdividef(g, 1.0f + __expf(-g)) * up[m];
         p.out[(size_t)m * p.out_ld + j] = a;
         const __nv_bfloat16 hi = __float2bfloat16_rn(a);
         p.out_hi[(size_t)m * p.out_ld + j] = hi;
