@@ -72,8 +72,11 @@ struct GemmCfg {
   static constexpr int TMEM_COLS = 2 * ACC_COLS;  // two accumulators
   static constexpr int NBAR = 2 * STAGES + 6;
   static constexpr int CS = MPAD * 64;           // EPI_QKV: RoPE (cos, sin) of every row and frequency
+  // residual rows loaded before the accumulator wait: every row up to 32 (MPAD 64 keeps
+  // the register budget with groups of EG)
+  static constexpr int EGR = MPAD <= 32 ? MPAD : EG;
   static constexpr size_t SMEM =
-      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 4 * 64 * 4 + CS * 8 + NBAR * 8 + 128;
+      1024 + (size_t)STAGES * STAGE_BYTES + STAGING * 4 + 2 * 64 * 4 + 64 * 8 + CS * 8 + NBAR * 8 + 128;
 };
 
 // First unit of CTA b's range.  The even split b*T/P moves back to the start of its tile
@@ -123,10 +126,11 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 
 template <int MPAD>
 __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, int r, float (&acc)[MPAD],
-                                               float* staging, const float* sinv, const int* s_slot, const int* s_seq,
-                                               const float (&pre)[EG], float pre_gn,
+                                               float* staging, const float* sinv, const long long* s_rowbase,
+                                               const float (&pre)[GemmCfg<MPAD>::EGR], float pre_gn,
                                                const float2* s_cs) {
   const int M = p.M;
+  constexpr int GR = GemmCfg<MPAD>::EGR;
   if (p.ssq_in) {
 #pragma unroll
     for (int m = 0; m < MPAD; ++m) acc[m] *= sinv[m];
@@ -138,13 +142,13 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int n = 128 * tile + r;
     const bool valid = n < p.N;
 #pragma unroll
-    for (int m0 = 0; m0 < MPAD; m0 += EG) {
-      float hv[EG];
+    for (int m0 = 0; m0 < MPAD; m0 += GR) {
+      float hv[GR];
 #pragma unroll
-      for (int u = 0; u < EG; ++u)
+      for (int u = 0; u < GR; ++u)
         hv[u] = m0 == 0 ? pre[u] : (m0 + u < M && valid) ? __ldcg(p.out + (size_t)(m0 + u) * p.out_ld + n) : 0.f;
 #pragma unroll
-      for (int u = 0; u < EG; ++u) {
+      for (int u = 0; u < GR; ++u) {
         const int m = m0 + u;
         if (m >= M) break;
         acc[m] = valid ? hv[u] + acc[m] : 0.f;   // h after the update
@@ -191,13 +195,13 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     if (n < p.N) {
       if (p.epi == EPI_RESID) {
 #pragma unroll
-        for (int m0 = 0; m0 < MPAD; m0 += EG) {
-          float hv[EG];
+        for (int m0 = 0; m0 < MPAD; m0 += GR) {
+          float hv[GR];
 #pragma unroll
-          for (int u = 0; u < EG; ++u)
+          for (int u = 0; u < GR; ++u)
             hv[u] = m0 == 0 ? pre[u] : (m0 + u < M) ? __ldcg(p.out + (size_t)(m0 + u) * p.out_ld + n) : 0.f;
 #pragma unroll
-          for (int u = 0; u < EG; ++u) acc[m0 + u] += hv[u];
+          for (int u = 0; u < GR; ++u) acc[m0 + u] += hv[u];
         }
       }
 #pragma unroll
@@ -215,14 +219,17 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
   // accumulators back from the exchange area instead of unrolling over MPAD rows.
   const float* mine = staging + r * (MPAD + 1);
   if (p.epi == EPI_SWIGLU) {
-    const int j = 64 * tile + r;
-    if (r < 64 && j < p.N) {
-      const float* up = staging + (r + 64) * (MPAD + 1);   // the up projection, lane r + 64
+    // 64 output columns per tile: column c pairs gate lane c with up lane c + 64; threads
+    // c and c + 64 take its even and odd rows
+    const int c = r & 63, j = 64 * tile + c;
+    if (j < p.N) {
+      const float* gate = staging + c * (MPAD + 1);
+      const float* up = staging + (c + 64) * (MPAD + 1);
       // SiLU through the fast exponential and division (a few ulp, far inside the tolerances
       // of an fp32 operand): the row loop is one dependent chain on the reducers' critical path
 #pragma unroll 1
-      for (int m = 0; m < M; ++m) {
-        const float g = mine[m];
+      for (int m = r >> 6; m < M; m += 2) {
+        const float g = gate[m];
         const float a = __fdividef(g, 1.0f + __expf(-g)) * up[m];
         p.out[(size_t)m * p.out_ld + j] = a;
         const __nv_bfloat16 hi = __float2bfloat16_rn(a);
@@ -244,21 +251,21 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const int partner = (i < half) ? r + half : r - half;
     const float* other = staging + partner * (MPAD + 1);
     const float sgn = (i < half) ? -1.f : 1.f;   // rotate-half RoPE: x cos -+ partner sin
-    __nv_bfloat16* cache = (which == 1) ? p.k_layer : p.v_layer;
+    __nv_bfloat16* cache = ((which == 1) ? p.k_layer : p.v_layer) + ((long long)head * p.cap * hd + i);
+    float* qout = p.out + f;
 #pragma unroll 1
-    for (int m = 0; m < M; ++m) {
+    for (int m = 0; m < M; ++m, qout += p.out_ld) {
       float val = mine[m];
       if (which < 2) {
         const float2 cs = s_cs[m * 64 + ih];
         val = val * cs.x + sgn * (other[m] * cs.y);
       }
       if (which == 0) {
-        p.out[(size_t)m * p.out_ld + f] = val;
+        *qout = val;
       } else {
-        const int slot = s_slot[m];
-        if (slot < p.cap) {
-          const int s = s_seq[m];
-          cache[(((size_t)s * p.H + head) * p.cap + slot) * hd + i] = __float2bfloat16_rn(val);
+        const long long base = s_rowbase[m];   // the row's cache element (seq, head 0, slot, 0)
+        if (base >= 0) {
+          cache[base] = __float2bfloat16_rn(val);
         } else if (i == 0 && which == 1) {
           set_error(p.err, ERR_CAPACITY);
         }
@@ -277,10 +284,11 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
   uint8_t* stages = smem;
   float* staging = reinterpret_cast<float*>(smem + (size_t)S * C::STAGE_BYTES);
   float* sinv = staging + C::STAGING;   // [64] RMSNorm row factors of the operand
-  int* s_slot = reinterpret_cast<int*>(sinv + 64);   // [64] EPI_QKV: cache slot of each row
-  int* s_pos = s_slot + 64;                          // [64] EPI_QKV: RoPE position of each row
-  int* s_seq = s_pos + 64;                           // [64] EPI_QKV: sequence of each row
-  float2* s_cs = reinterpret_cast<float2*>(s_seq + 64);   // [MPAD][64] EPI_QKV: RoPE factors
+  int* s_pos = reinterpret_cast<int*>(sinv + 64);    // [64] EPI_QKV: RoPE position of each row
+  // [64] EPI_QKV: offset of each row's cache element (sequence, head 0, slot, dimension 0),
+  // -1 past the capacity (8-byte aligned: the area before is a multiple of 8 bytes)
+  long long* s_rowbase = reinterpret_cast<long long*>(s_pos + 64);
+  float2* s_cs = reinterpret_cast<float2*>(s_rowbase + 64);   // [MPAD][64] EPI_QKV: RoPE factors
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_cs + C::CS);
   uint64_t* full = bars;             // weights and activations of the stage landed (TMA)
   uint64_t* empty = bars + S;        // stage consumed by the tensor core
@@ -449,9 +457,8 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
           set_error(p.err, ERR_POSITION);
           pos = pos < 0 ? 0 : p.rope_len - 1;
         }
-        s_slot[r] = slot;
         s_pos[r] = pos;
-        s_seq[r] = seq;
+        s_rowbase[r] = slot < p.cap ? ((long long)seq * p.H * p.cap + slot) * p.hd : -1;
       }
       named_bar_sync(1, 128);
       // the RoPE factors of every row, in shared memory long before any accumulator is ready
@@ -485,13 +492,13 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
       const int buf = seg & 1;
       // what this tile's epilogue reads from global memory (first row group), loaded while
       // the tensor cores work: residual rows and gain
-      float pre[EG];
+      float pre[C::EGR];
       float pre_gn = 0.f;
       {
         const int n = 128 * tile + r;
         const bool resid = p.epi == EPI_RESID && n < p.N;
 #pragma unroll
-        for (int u = 0; u < EG; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
+        for (int u = 0; u < C::EGR; ++u) pre[u] = (resid && u < p.M) ? __ldcg(p.out + (size_t)u * p.out_ld + n) : 0.f;
         if (resid && p.gain_next) pre_gn = __bfloat162float(p.gain_next[n]);
       }
       // the four epilogue warps decide together (lanes leave the polling loop at different
@@ -582,7 +589,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         if (r == 0) p.counters[tile] = 0;
       }
       if (r == 0 && last_seg && p.trace.rec) s_mark[2] = globaltimer_ns();
-      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_slot, s_seq, pre, pre_gn, s_cs);
+      epilogue_final<MPAD>(p, tile, r, acc, staging, sinv, s_rowbase, pre, pre_gn, s_cs);
     }
   }
 
