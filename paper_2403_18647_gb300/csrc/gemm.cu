@@ -253,7 +253,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
     const float sgn = (i < half) ? -1.f : 1.f;   // rotate-half RoPE: x cos -+ partner sin
     __nv_bfloat16* cache = ((which == 1) ? p.k_layer : p.v_layer) + ((long long)head * p.cap * hd + i);
     float* qout = p.out + f;
-#pragma unroll 1
+#pragma unroll 2   // two rows in flight (4 made the cold loop slower)
     for (int m = 0; m < M; ++m, qout += p.out_ld) {
       float val = mine[m];
       if (which < 2) {
@@ -484,6 +484,8 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
         s_share[3 * i + 2] = unit_begin(lo, T, p.P, p.kc, p.snap) == t * p.kc ? 0 : 1;
       }
     }
+    // partials per bulk-copy round of the last reducer (the idle stage ring holds them)
+    const int red_per = max(1, (int)((S * C::STAGE_BYTES) / ((uint32_t)p.M * 512)));
     int seg = 0, tile = tile_first - 1;
     long long g = g0;
     while (g < g1) {
@@ -551,7 +553,7 @@ __global__ void __launch_bounds__(192, SDSAT_GEMM_MINB) gemm_kernel(const __grid
           // The stage ring is idle after the CTA's last tile (every TMA load landed and every
           // MMA that read it completed): bulk-copy the contributors' partials into it, as many
           // per round as fit, and sum them in CTA order.
-          const int per = max(1, (int)((S * C::STAGE_BYTES) / pbytes));
+          const int per = red_per;
           const float* ring = reinterpret_cast<const float*>(stages);
           uint32_t ph = 0;
           bool ok = true;
