@@ -304,58 +304,9 @@ struct NucList {
   int id[NUC_LIST_MAX];
   uint32_t cnt[NUC_FLOORS];                 // block totals: weights >= floor f
   unsigned long long mhi[3], mlo[3];        // masses >= floors 4, 5, 6: sum(w >> 12), sum(w & 4095)
+  unsigned long long kstar, sk;             // the kept prefix's last key and its mass
   int pick;
 };
-
-// warp-wide sums: per-lane values below 2^32 (counts, or weights of <= 128 list elements)
-__device__ __forceinline__ uint64_t warp_sum_w(uint32_t v) {
-  const uint32_t hi = __reduce_add_sync(0xffffffffu, v >> 16), lo = __reduce_add_sync(0xffffffffu, v & 0xFFFFu);
-  return ((uint64_t)hi << 16) + lo;
-}
-
-// over the list: sum of W (COUNT: number of elements) of those with pred(W, id)
-template <bool COUNT, typename F>
-__device__ __forceinline__ uint64_t list_sum(const NucList& L, int n, F&& pred) {
-  uint32_t s = 0;
-  for (int i = (int)(threadIdx.x & 31); i < n; i += 32) {
-    const uint32_t w = L.w[i];
-    if (pred(w, L.id[i])) s += COUNT ? 1u : w;
-  }
-  return warp_sum_w(s);
-}
-
-// largest x in [0, 2^24] with list_sum(pred_x) >= need, pred_x(w, id) = sel(w, id) && w >= x
-template <bool COUNT, typename F>
-__device__ __forceinline__ uint32_t list_threshold(const NucList& L, int n, uint64_t need, F&& sel) {
-  uint32_t lo = 0, hi = 1u << 24;
-  while (lo < hi) {
-    const uint32_t mid = lo + (hi - lo + 1) / 2;
-    if (list_sum<COUNT>(L, n, [&](uint32_t w, int id) { return w >= mid && sel(w, id); }) >= need) lo = mid;
-    else hi = mid - 1;
-  }
-  return lo;
-}
-
-// id of the r-th (r >= 1) list element, in list (= ascending id) order, with pred(W, id)
-template <typename F>
-__device__ __forceinline__ int list_nth(const NucList& L, int n, uint64_t r, F&& pred) {
-  const int lane = threadIdx.x & 31;
-  uint64_t seen = 0;
-  for (int b = 0; b < n; b += 32) {
-    const int i = b + lane;
-    const bool hit = i < n && pred(L.w[i], L.id[i]);
-    const uint32_t m = __ballot_sync(0xffffffffu, hit);
-    const uint32_t c = __popc(m);
-    if (seen + c >= r) {
-      const int k = (int)(r - seen);      // the k-th set bit of m
-      uint32_t mm = m;
-      for (int t = 1; t < k; ++t) mm &= mm - 1;
-      return __shfl_sync(0xffffffffu, L.id[b + __ffs(mm) - 1 < n ? b + __ffs(mm) - 1 : 0], 0);
-    }
-    seen += c;
-  }
-  return 0x7FFFFFFF;
-}
 
 __device__ __forceinline__ uint64_t nuc_key(uint32_t w, int id) {   // larger: heavier, then lower id
   return ((uint64_t)w << 32) | (uint32_t)(0x7FFFFFFF - id);
@@ -421,56 +372,98 @@ __device__ int list_small(const AcceptParams& p, const NucList& L, int n, uint64
   return __shfl_sync(0xffffffffu, id, __ffs(m) - 1);
 }
 
-// steps 4-7 of the sampler on the list (warp 0): candidates, kept set, draw, pick.  S_all is
-// the mass of every id (the candidates' mass when there is no top-k).
-__device__ int list_select(const AcceptParams& p, const NucList& L, int n, uint64_t S_all, uint64_t rnd) {
-  const int lane = threadIdx.x & 31;
-  // 4. top-k candidates: W > xk, or W == xk and id <= idk
-  uint32_t xk = 0;
-  int idk = 0x7FFFFFFF;
-  const bool topk = p.top_k > 0 && p.top_k < p.V;
-  if (topk && n >= p.top_k) {
-    const uint64_t k = (uint64_t)p.top_k;
-    xk = list_threshold<true>(L, n, k, [](uint32_t, int) { return true; });
-    const uint64_t above = list_sum<true>(L, n, [&](uint32_t w, int) { return w > xk; });
-    idk = list_nth(L, n, k - above, [&](uint32_t w, int) { return w == xk; });
+// Steps 4-7 on the list with the whole block.  The list holds the first n elements of the
+// order (W desc, id asc) in ascending id; its keys are sorted once (bitonic, descending, over
+// the list's own storage), so the candidates (the first min(k, n)), their mass, the kept
+// prefix (the shortest one whose mass reaches ceil(P S / 2^24)) and its mass are prefix sums
+// of the sorted weights.  The pick then scans every id's weight, still in registers, in
+// ascending id with "kept" = key >= the kept prefix's last key.
+__device__ int list_sorted_select(const AcceptParams& p, NucList& L, int n, uint64_t S_all, uint64_t rnd,
+                                  const uint32_t (&W)[ACC_EPT], int base, uint64_t* red, int* redi) {
+  constexpr int PER = NUC_LIST_MAX / ACC_THREADS;   // list elements per thread
+  uint64_t* K = reinterpret_cast<uint64_t*>(L.w);    // NUC_LIST_MAX keys over w[] and id[]
+  int n2 = 32;
+  while (n2 < n) n2 <<= 1;
+  uint64_t kk[PER];
+#pragma unroll
+  for (int r = 0; r < PER; ++r) {
+    const int i = threadIdx.x + r * ACC_THREADS;
+    kk[r] = i < n ? nuc_key(L.w[i], L.id[i]) : 0ull;   // padding sorts last (every list W >= 1)
   }
-  // (n < k: the list holds every non-zero weight, all of them candidates; the zero-weight
-  // candidates add nothing to any sum and are never kept)
-  auto cand = [&](uint32_t w, int id) { return w > xk || (w == xk && id <= idk); };
-  // 5. top-p over the candidates
-  const uint64_t S = topk ? list_sum<false>(L, n, cand) : S_all;
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < PER; ++r) {
+    const int i = threadIdx.x + r * ACC_THREADS;
+    if (i < n2) K[i] = kk[r];
+  }
+  __syncthreads();
+  for (int k = 2; k <= n2; k <<= 1)
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < n2; i += ACC_THREADS) {
+        const int l = i ^ j;
+        if (l > i) {
+          const uint64_t a = K[i], b = K[l];
+          if (((i & k) == 0) == (a < b)) {   // descending blocks where bit k of i is clear
+            K[i] = b;
+            K[l] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  // candidates and the kept prefix: thread t holds sorted elements PER*t .. PER*t + PER - 1
+  const bool topk = p.top_k > 0 && p.top_k < p.V;
+  const int nc = topk ? min(p.top_k, n) : n;
+  const int i0 = threadIdx.x * PER;
+  uint64_t wsum = 0;
+#pragma unroll
+  for (int e = 0; e < PER; ++e)
+    if (i0 + e < nc) wsum += K[i0 + e] >> 32;
+  const uint64_t S = topk ? block_sum_u64(wsum, red) : S_all;
   const uint64_t prod = (uint64_t)p.p_fixed * S;
   const uint64_t thr = (prod >> 24) + ((prod & 0xFFFFFFull) ? 1 : 0);
-  uint32_t xp = 0;
-  int idp = -1;   // thr >= S: every non-zero candidate is kept
-  if (thr < S) {
-    xp = list_threshold<false>(L, n, thr, cand);
-    const uint64_t above = list_sum<false>(L, n, [&](uint32_t w, int id) { return cand(w, id) && w > xp; });
-    const uint64_t n_above = list_sum<true>(L, n, [&](uint32_t w, int id) { return cand(w, id) && w > xp; });
-    uint64_t ties = thr > above ? (thr - above + xp - 1) / xp : 0;
-    if (n_above == 0 && ties == 0) ties = 1;
-    idp = ties == 0 ? -1 : list_nth(L, n, ties, [&](uint32_t w, int id) { return cand(w, id) && w == xp; });
-  }
-  auto kept = [&](uint32_t w, int id) { return cand(w, id) && (w > xp || (w == xp && id <= idp)); };
-  const uint64_t Sk = list_sum<false>(L, n, kept);
-  // 6. the draw, 7. the first kept id whose inclusive cumulative weight exceeds tau
-  const uint64_t tau = __umul64hi(rnd, Sk);
-  uint64_t carry = 0;
-  for (int b = 0; b < n; b += 32) {
-    const int i = b + lane;
-    const uint32_t w = (i < n && kept(L.w[i], L.id[i])) ? L.w[i] : 0u;
-    uint32_t x = w;   // inclusive prefix within the chunk (< 2^29)
+  const uint64_t before = block_exscan_u64(wsum, red);
+  // the first sorted index whose inclusive mass reaches thr (index 0 when thr = 0); the list
+  // provably holds it
+  if (thr == 0 ? threadIdx.x == 0 : (before < thr && before + wsum >= thr)) {
+    uint64_t cum = before;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
-      if (lane >= o) x += y;
+    for (int e = 0; e < PER; ++e) {
+      cum += K[i0 + e] >> 32;
+      if (cum >= thr) {
+        L.kstar = K[i0 + e];
+        L.sk = cum;
+        break;
+      }
     }
-    const uint32_t m = __ballot_sync(0xffffffffu, w != 0 && carry + x > tau);
-    if (m) return __shfl_sync(0xffffffffu, L.id[b + __ffs(m) - 1], 0);
-    carry += __shfl_sync(0xffffffffu, x, 31);
   }
-  return 0x7FFFFFFF;   // not reached: tau < Sk
+  __syncthreads();
+  const uint64_t kstar = L.kstar, Sk = L.sk;
+  const uint64_t tau = __umul64hi(rnd, Sk);
+  // 7. the first kept id (ascending) whose inclusive cumulative weight exceeds tau
+  uint64_t mine = 0;
+#pragma unroll
+  for (int e = 0; e < ACC_EPT; ++e)
+    if (nuc_key(W[e], base + e) >= kstar) mine += W[e];
+  const uint64_t below = block_exscan_u64(mine, red);
+  if (threadIdx.x == 0) redi[0] = 0x7FFFFFFF;
+  __syncthreads();
+  if (below <= tau && below + mine > tau) {
+    uint64_t cum = below;
+    int pick = 0x7FFFFFFF;
+#pragma unroll
+    for (int e = 0; e < ACC_EPT; ++e) {
+      if (nuc_key(W[e], base + e) >= kstar) {
+        cum += W[e];
+        if (cum > tau && pick == 0x7FFFFFFF) pick = base + e;
+      }
+    }
+    redi[0] = pick;
+  }
+  __syncthreads();
+  const int out = redi[0];
+  __syncthreads();
+  return out;
 }
 
 __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* row, int position, int seq,
@@ -597,13 +590,18 @@ __device__ __forceinline__ int row_nucleus(const AcceptParams& p, const float* r
           ++at;
         }
       __syncthreads();
-      if (w == 0) {
-        int pick = list_small(p, L, N[f], S_all, topk, rnd);
-        if (pick < 0) pick = list_select(p, L, N[f], S_all, rnd);
-        if (lane == 0) L.pick = pick;
+      // a kept set (or top-k) of at most 32 on the lanes of one warp when that is cheap: a
+      // small top-k, or a short list; otherwise, or when it does not apply, the sorted list
+      if ((topk && p.top_k <= 32) || N[f] <= 64) {
+        if (w == 0) {
+          const int pick = list_small(p, L, N[f], S_all, topk, rnd);
+          if (lane == 0) L.pick = pick;
+        }
+        __syncthreads();
+        const int pick = L.pick;
+        if (pick >= 0) return pick;
       }
-      __syncthreads();
-      return L.pick;
+      return list_sorted_select(p, L, N[f], S_all, rnd, W, base, red, redi);
     }
   }
 
