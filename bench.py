@@ -59,13 +59,13 @@ WORKLOADS = {
 
 
 # DRAM bytes (read + write) per algorithmic byte of the skinny GEMM, from one ncu capture
-# (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.02 MB of traffic for
+# (--set full) of a gate/up-sized launch: K 4096, N 22016, M 6 -> 186.01 MB of traffic for
 # 180.98 MB of weights + operand + output.  The bench line applies it to the step's gate/up
 # launch (the roofline's kernel).  GEMM_TRAFFIC_CURRENT says whether that capture was taken of
 # the kernel as it is now; while it is False the line reports traffic null.
-GEMM_TRAFFIC_RATIO = 186.02 / 180.98
-GEMM_TRAFFIC_CURRENT = False
-GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.02 MB for 180.98 MB "
+GEMM_TRAFFIC_RATIO = 186.01 / 180.98
+GEMM_TRAFFIC_CURRENT = True
+GEMM_TRAFFIC_SOURCE = ("ncu dram__bytes_read+write of one K=4096 N=22016 M=6 launch (186.01 MB for 180.98 MB "
                        "algorithmic, profiles/gemm_gateup_4096x22016_m6.md) times the gate/up launch's algorithmic "
                        "bytes; bytes per launch")
 

@@ -272,6 +272,43 @@ def test_accept_nucleus_full_vocab(sd):
         assert out == rout and acc == racc
 
 
+def _sorted_list_rows(V, sizes, seed):
+    """Rows whose heavy set has exactly n ids (the rest at -100, weight 0): tied logit values
+    for even rows, a narrow continuum for odd ones, so that kept sets of more than 32 take
+    the sampler's sorted-list path at list sizes that are not powers of two."""
+    g = torch.Generator().manual_seed(seed)
+    rows = []
+    for i, n in enumerate(sizes):
+        r = torch.full((V,), -100.0)
+        ids = torch.randperm(V, generator=g)[:n]
+        if i % 2 == 0:
+            vals = torch.tensor([0.0, -0.05, -0.1, -0.2])[torch.randint(0, 4, (n,), generator=g)]
+        else:
+            vals = torch.randn(n, generator=g) * 0.5
+        r[ids] = vals
+        rows.append(r)
+    return torch.stack(rows).float()
+
+
+@pytest.mark.parametrize("T,top_p,top_k", [(1.0, 0.95, 0), (0.2, 0.95, 0), (1.0, 0.9, 100), (1.0, 0.999, 0)])
+def test_accept_nucleus_sorted_list_sizes(sd, T, top_p, top_k):
+    """The sorted-list path (kept sets beyond 32, lists of 65-4096) on a 32016-entry vocabulary:
+    bit-exact against the oracle, ties in W included."""
+    big = synth.ModelShape("v32k", 1, 256, 4, 64, 688, 32016, 32011)
+    w = synth.make_model(big, seed=0, device="cuda")
+    ctx = sd.Context(big, w, max_position=4096)
+    sizes = [65, 100, 257, 690, 1000, 1023, 1025, 2049, 3000, 4000, 4096, 130, 513, 777]
+    b, q = 2, 7
+    lg = _sorted_list_rows(32016, sizes, 31 + int(T * 10) + top_k)
+    lgc = lg.numpy()
+    lens = [300, 2000]
+    acc, out, flags, _ = _run_accept(ctx, lg.cuda(), torch.zeros(b * q, dtype=torch.int32, device="cuda"), b, q, 0,
+                                     lens, T, top_p, 5, top_k)
+    _, rout = _oracle_accept(lgc, [0] * (b * q), b, q, 0, lens, T, top_p, 5, top_k)
+    assert out == rout
+    assert flags == 0
+
+
 def _nucleus_rows(V):
     """Rows that steer the sampler's list path (heavy weights compacted, at each floor) and its
     block-wide path (too many heavy weights), at the boundaries between them."""
