@@ -20,7 +20,7 @@
 // two-stage ring of K and V tiles (TMA, boxes of 64 dims x 64 rows, 128-byte
 // swizzle) full, walking the CTA's units pair by pair; tiles made of committed
 // slots only are requested before the QKV projection has finished, and the
-// next ATT_PREFETCH tiles are kept on their way into L2.  Per unit, on the
+// next ATT_PREFETCH tiles (one for long slices) are kept on their way into L2.  Per unit, on the
 // tensor cores (mma.sync m16n8k16) in transposed form, so that the q <= 8
 // block rows fill an N = 8 tile instead of padding an M = 16 one: S^T = K Q^T
 // with each warp on 16 keys, an online-softmax update of the running row max
@@ -46,6 +46,13 @@ namespace sdsat {
 
 constexpr int ATT_STAGES = 2;
 constexpr int ATT_PREFETCH = 4;   // units past the ring requested into L2 ahead of their loads
+// ... but only one for a CTA whose slice has at least this many units.  Thread 0 issues the
+// window before the dependency wait, and the TMA unit works through the requests of the SM's
+// three CTAs in order: with long slices (13B at context 4096: 7-8 units) thread 0 reached the
+// wait 2.8 us after the QKV projection ended with a window of 4 (1.0 us with 1; 13B forward
+// 5.303 -> 5.256 ms), while shorter slices (batch 4 at context 1024: 5-6 units) lose more from
+// the later units' missed L2 hits than they gain (attention 13.7 -> 15.1 us with 1)
+constexpr int ATT_LONG_SLICE = 7;
 constexpr int ATT_SPARE_CLUSTERS = 8;   // room left for this many more clusters (measured: 7B/13B shapes, b = 1, 4)
 
 template <int HD, int QT = 2>
@@ -216,7 +223,10 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
     }
     pfc = isu;
     for (int k = issued; k < ATT_STAGES && pfc.pi < npairs; ++k) advance(pfc);
-    for (int k = 0; k < ATT_PREFETCH && pfc.pi < npairs; ++k) {
+    int cb0 = 0, ce0 = 0;
+    if (cl < npairs) slice(cl, cb0, ce0);
+    const int window = ce0 - cb0 >= ATT_LONG_SLICE ? 1 : ATT_PREFETCH;
+    for (int k = 0; k < window && pfc.pi < npairs; ++k) {
       bool committed;
       const int row = unit_row(pfc, committed);
       if (committed) prefetch(row);
