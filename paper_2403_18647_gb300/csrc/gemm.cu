@@ -43,7 +43,6 @@ namespace sdsat {
 #ifndef SDSAT_GEMM_STAGES16
 #define SDSAT_GEMM_STAGES16 4
 #endif
-// Minimum resident CTAs per SM the register allocation must allow (192 threads each).
 // Stream-K split points within the first SDSAT_GEMM_SNAP units of a tile move to the tile's
 // start, for GEMMs with at least SDSAT_GEMM_SNAP_MIN_UNITS units per CTA.
 #ifndef SDSAT_GEMM_SNAP
@@ -52,6 +51,7 @@ namespace sdsat {
 #ifndef SDSAT_GEMM_SNAP_MIN_UNITS
 #define SDSAT_GEMM_SNAP_MIN_UNITS 24
 #endif
+// Minimum resident CTAs per SM the register allocation must allow (192 threads each).
 #ifndef SDSAT_GEMM_MINB
 #define SDSAT_GEMM_MINB 2
 #endif
@@ -240,7 +240,7 @@ __device__ __forceinline__ void epilogue_final(const GemmParams& p, int tile, in
   } else {  // EPI_QKV
     // This runs once per launch on the reducers' critical path, so no division: the
     // projection by comparison, head and dimension by shift and mask (hd is 64 or 128), and
-    // each row's sequence from the table the setup filled.
+    // each row's cache offset from the table the setup filled.
     const int R = p.rows_per_map;
     const int gf = 128 * tile + r;
     const int which = (gf >= R) + (gf >= 2 * R);
