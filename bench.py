@@ -717,6 +717,7 @@ def run_e2e(r, steps, steps_per_gen):
     runs the step's calls (block_forward and accept; a tree step: the tree forward and tree
     accept) as one CUDA-graph replay, copies the emitted tokens and accepted lengths back and
     reads them before the next step."""
+    import numpy as np
     import torch
     b, k = r.b, r.k
     qm = r.qmax
@@ -738,6 +739,10 @@ def run_e2e(r, steps, steps_per_gen):
     st = torch.cuda.current_stream()
     if r.pipe:
         return run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start, fns[1], how)
+    # the host side works on numpy views of the pinned buffers (no per-step allocations)
+    tok_np, out_np, acc_np = tok_h.numpy(), out_h.numpy(), acc_h.numpy()
+    table_np = table.numpy()
+    adaptive_np = np.asarray(adaptive, dtype=np.int32)
     t0 = time.perf_counter()
     for i in range(steps):
         j = i % steps_per_gen
@@ -746,26 +751,24 @@ def run_e2e(r, steps, steps_per_gen):
             lens, last_out, last_acc = start()
         mode = 1 if j % 2 == 0 else 2
         q = r.q if mode == 1 else r.q2
-        blk = []
         for s in range(b):
             if mode == 1:
-                blk += [last_out[s][last_acc[s] - 1]] + adaptive
+                tok_np[s * q] = last_out[s][last_acc[s] - 1]
+                tok_np[s * q + 1:s * q + q] = adaptive_np
             else:
-                blk += [last_out[s][0]] + [int(table[w, s, lens[s] + jj]) for w in range(r.width)
-                                           for jj in range(1, k + 1)]
-        tok_h[:b * q].copy_(torch.tensor(blk, dtype=torch.int32))
+                tok_np[s * q] = last_out[s][0]
+                for w in range(r.width):
+                    tok_np[s * q + 1 + w * k:s * q + 1 + (w + 1) * k] = table_np[w, s, lens[s] + 1:lens[s] + k + 1]
         r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
         fns[mode]()
         out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
         acc_h.copy_(r.acc, non_blocking=True)
         st.synchronize()
-        o = out_h.tolist()
-        a = acc_h.tolist()
         for s in range(b):
-            last_out[s] = o[s * q:(s + 1) * q]
-            last_acc[s] = a[s]
-            lens[s] += a[s]
-        tokens += sum(a)
+            last_out[s] = out_np[s * q:(s + 1) * q].copy()
+            last_acc[s] = int(acc_np[s])
+            lens[s] += last_acc[s]
+        tokens += int(acc_np.sum())
         h2d += b * q * 4
         d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
@@ -776,9 +779,14 @@ def run_e2e(r, steps, steps_per_gen):
 def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adaptive, start, fn, how):
     """run_e2e for the pipelined variant: the host keeps each sequence's block mode, builds
     [x_0, drafts or adaptive ids, adaptive ids] and copies the per-sequence verify counts in."""
+    import numpy as np
     import torch
     b, k, q = r.b, r.k, r.q
     nv_h = torch.zeros(b, dtype=torch.int32).pin_memory()
+    # the host side works on numpy views of the pinned buffers (no per-step allocations)
+    tok_np, out_np, acc_np, nv_np = tok_h.numpy(), out_h.numpy(), acc_h.numpy(), nv_h.numpy()
+    table_np = table.numpy()
+    adaptive_np = np.asarray(adaptive, dtype=np.int32)
     lens, last_out, last_acc = start()
     prev_mode = [1] * b
     tokens = h2d = d2h = 0
@@ -789,28 +797,24 @@ def run_e2e_pipelined(r, steps, steps_per_gen, tok_h, out_h, acc_h, table, adapt
             r.reset()
             lens, last_out, last_acc = start()
             prev_mode = [1] * b
-        blk, nv = [], []
         for s in range(b):
             a_mode = prev_mode[s] == 0 or last_acc[s] == k + 1
-            x0 = last_out[s][last_acc[s] - 1]
-            mid = [int(table[0, s, lens[s] + jj]) for jj in range(1, k + 1)] if a_mode else adaptive
-            blk += [x0] + mid + adaptive
-            nv.append(k if a_mode else 0)
+            tok_np[s * q] = last_out[s][last_acc[s] - 1]
+            tok_np[s * q + 1:s * q + 1 + k] = table_np[0, s, lens[s] + 1:lens[s] + k + 1] if a_mode else adaptive_np
+            tok_np[s * q + 1 + k:s * q + 1 + 2 * k] = adaptive_np
+            nv_np[s] = k if a_mode else 0
             prev_mode[s] = 1 if a_mode else 0
-        tok_h[:b * q].copy_(torch.tensor(blk, dtype=torch.int32))
-        nv_h.copy_(torch.tensor(nv, dtype=torch.int32))
         r.toks[:b * q].copy_(tok_h[:b * q], non_blocking=True)
         r.pnver.copy_(nv_h, non_blocking=True)
         fn()
         out_h[:b * q].copy_(r.out[:b * q], non_blocking=True)
         acc_h.copy_(r.acc, non_blocking=True)
         st.synchronize()
-        o, a = out_h.tolist(), acc_h.tolist()
         for s in range(b):
-            last_out[s] = o[s * q:(s + 1) * q]
-            last_acc[s] = a[s]
-            lens[s] += a[s]
-        tokens += sum(a)
+            last_out[s] = out_np[s * q:(s + 1) * q].copy()
+            last_acc[s] = int(acc_np[s])
+            lens[s] += last_acc[s]
+        tokens += int(acc_np.sum())
         h2d += b * q * 4 + b * 4
         d2h += b * q * 4 + b * 4
     t1 = time.perf_counter()
