@@ -479,7 +479,11 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
     cluster_sync_all();   // the cluster's cs partials of the pair are complete
     // ---- merge this CTA's share of the pair's (row, 4 dimensions) outputs over the cs
     // partials, read in rank order from the cluster's shared memory: w_r = exp(m_r - max m),
-    // L = sum_r w_r l_r, O = (sum_r w_r o_r) / L
+    // L = sum_r w_r l_r, O = (sum_r w_r o_r) / L.  The second cluster barrier only keeps the
+    // partials in place until every CTA has read them, so each thread arrives at it right
+    // after its last remote loads and waits only at the end: the barrier's round trip
+    // overlaps the merge arithmetic and the output stores.
+    bool arrived = false;
     {
       const int items = q * D4, i0 = items * rank / CS, i1 = items * (rank + 1) / CS;
       for (int it = i0 + tid; it < i1; it += 128) {
@@ -493,6 +497,10 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
             ml[r] = ld_dsmem_f2(mapa_shared(a_ml, r));
             ov[r] = ld_dsmem_f4(mapa_shared(a_o, r));
           }
+        if (it + 128 >= i1) {   // this thread's last item: its reads of the partials are done
+          cluster_arrive_thread();
+          arrived = true;
+        }
         float mx = -INFINITY;
 #pragma unroll
         for (int r = 0; r < ATT_CS_MAX; ++r)
@@ -526,7 +534,8 @@ __global__ void __launch_bounds__(128, QT == 1 ? 3 : 1) attention_kernel(const _
     }
     if (p.trace.rec) t_merge = globaltimer_ns();
     ++pairs_done;
-    cluster_sync_all();   // every CTA of the cluster has read this CTA's partial
+    if (!arrived) cluster_arrive_thread();   // a thread without an item to merge
+    cluster_wait_thread();   // every CTA of the cluster has read this CTA's partial
   }
   if (*abort_flag && tid == 0) {   // let the copies in flight land before the CTA exits
     for (int i = max(0, issued - ATT_STAGES); i < issued; ++i) {

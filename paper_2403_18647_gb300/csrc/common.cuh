@@ -55,6 +55,14 @@ __device__ __forceinline__ void cluster_sync_all() {
   __syncwarp();   // the .aligned forms want the whole warp converged
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// the two halves of a cluster barrier, per thread (not .aligned: the threads of a warp may
+// arrive at different points); every thread of the cluster arrives once, then waits once
+__device__ __forceinline__ void cluster_arrive_thread() {
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_thread() {
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+}
 // the address of the same shared-memory location in the CTA of the cluster with rank `rank`
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   uint32_t r;
