@@ -365,6 +365,24 @@ def test_gemm_13b_shapes_sampled(tiny_ctx, N, K):
     assert err <= 5e-5 * math.sqrt(K) * 0.02 + 1e-6 * np.abs(ref).max(), err
 
 
+@pytest.mark.parametrize("M", [6, 24])
+@pytest.mark.parametrize("K,N", [(2048, 49152), (3072, 24576), (4096, 16384)])
+def test_gemm_streamk_snapped_full(tiny_ctx, M, K, N):
+    """Shapes whose stream-K split gives every CTA >= 24 units (304 CTAs on GB300), so split
+    points that land in a tile's first 3 units move to the tile's start (16-32 of them here),
+    at the two operand widths (M = 6: MPAD 16; M = 24: MPAD 32): every output element against
+    fp64 dot products, so every tile's contributor set and partial slots are exercised."""
+    x = synth.normal_f32(6, M * 7 + K, (M, K), 1.0, device="cuda")
+    w = synth.normal_bf16(6, N + K, (N, K), 0.02, device="cuda")
+    y = torch.empty((M, N), device="cuda")
+    tiny_ctx.op_gemm(x, w, y)
+    torch.cuda.synchronize()
+    ref = OM.linear(x.cpu().double().numpy(), w.cpu().double().numpy())
+    err = np.abs(y.cpu().double().numpy() - ref).max()
+    assert err <= 5e-5 * math.sqrt(K) * 0.02 + 1e-6 * np.abs(ref).max(), err
+    assert tiny_ctx.get_error() == 0
+
+
 def test_attention_40_heads_sampled(big_ctx):
     """40 heads (the 13B shape) at context 4096, q = 6: three sampled heads against the oracle."""
     b, q, H, hd, n = 1, 6, 40, 128, 4096
